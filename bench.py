@@ -1,0 +1,411 @@
+"""Decode-step benchmark: paged decode attention (+ fused K/V append) on GB300.
+
+A step is one pass of the whole hot path over one batch: kv_begin_step (lazy
+page allocation, page-table update and split plan on the device) and, for each
+of the L layers, kv_append then decode_attention.  The default workload is the
+LLaVA-1.5-7B-shaped batch (32 layers, 32/32 heads, d 128, batch 64, 576 vision
+tokens + U[64,512] prompt + U{0..256} generated tokens, page 16, shuffled page
+table).  Inputs are seeded synthetic draws (paper_2603_12707_gb300.workloads).
+
+value = algorithmic bytes of the K timed steps / their device time (GB/s):
+per layer and sequence, K and V of every attended token, the Q read, the O
+write and the appended K/V write, all bf16.  The roofline object reports the
+decode_attention kernel alone (KV + Q + O bytes per launch over its CUDA-event
+duration on the launch stream) against the measured HBM copy bandwidth.
+
+Multi-GPU: the path has no exchange step, so N GPUs run N independent replicas
+(weak scaling); ranks meet only for the barrier and the max of their times.
+--impl reference times the float64 CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-attention achieved HBM GB/s (% of GB300 peak) and decode steps/sec"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def layer_bytes(cfg, attended):
+    """(attention bytes, append bytes) of one layer: KV of every attended
+    token + Q read + O write; appended K and V written."""
+    Hq, Hkv, d = cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+    B = len(attended)
+    attn = int(sum(attended)) * 2 * Hkv * d * 2 + B * Hq * d * 2 * 2
+    app = B * 2 * Hkv * d * 2
+    return attn, app
+
+
+def describe(cfg):
+    return {"workload": cfg.name + ": " + cfg.description, "batch": cfg.batch, "layers": cfg.num_layers,
+            "layer_pools": cfg.phys_layers, "q_heads": cfg.num_q_heads, "kv_heads": cfg.num_kv_heads,
+            "head_dim": cfg.head_dim, "page_size": cfg.page_size, "seed": cfg.seed}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception as e:  # no nvidia-smi: report no samples
+            log("clock sampling unavailable:", e)
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_smi_id(torch, dev):
+    try:
+        p = torch.cuda.get_device_properties(dev)
+        return f"{p.pci_domain_id:08X}:{p.pci_bus_id:02X}:{p.pci_device_id:02X}.0"
+    except Exception:
+        return str(dev)
+
+
+# --------------------------------------------------------- kernel traffic
+def committed_traffic(kernel_src):
+    """DRAM bytes per launch of the decode kernel from the committed ncu
+    summary, valid only if it was taken on the current kernel source."""
+    p = os.path.join(ROOT, "profiles", "decode_kernel_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    with open(kernel_src, "rb") as f:
+        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    return d if d.get("source_sha256_16") == h else None
+
+
+# ------------------------------------------------------------- CPU oracle
+def oracle_sample(cfg, budget_s):
+    """Time the float64 oracle on one layer of the workload (all sequences and
+    heads, one decode step), repeated until about budget_s seconds of oracle
+    time or one full step's worth of layers.  Returns (bytes, seconds,
+    description, threads)."""
+    import oracle
+    from paper_2603_12707_gb300 import workloads as wl
+    import torch
+    lens = [int(n) + 1 for n in wl.context_lengths(cfg)]
+    k = torch.cat([wl.kv_block(cfg, 0, b, n, "k", "cpu") for b, n in enumerate(lens)])
+    v = torch.cat([wl.kv_block(cfg, 0, b, n, "v", "cpu") for b, n in enumerate(lens)])
+    q = wl.step_inputs(cfg, 0, 0, "cpu")[0]
+    attn, _ = layer_bytes(cfg, lens)
+    done_bytes, spent, layers = 0, 0.0, 0
+    while spent < budget_s and layers < cfg.num_layers:
+        t0 = time.perf_counter()
+        oracle.decode_attention(q, lens, k, v)
+        spent += time.perf_counter() - t0
+        done_bytes += attn
+        layers += 1
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    desc = (f"{layers} of {cfg.num_layers} layers of one decode step of the {cfg.name} workload "
+            f"({cfg.batch} sequences x {cfg.num_q_heads} heads each; every layer repeats layer 0's K/V), "
+            f"float64 oracle, OpenMP over (sequence, head)")
+    return done_bytes, spent, desc, threads
+
+
+# -------------------------------------------------------------- GPU run
+def run_gpu(args, rank, world):
+    import torch
+    from paper_2603_12707_gb300 import _build, kvdecode as kd, workloads as wl
+    from paper_2603_12707_gb300.harness import DecodeSession
+
+    dev = int(os.environ.get("LOCAL_RANK", 0))
+    torch.cuda.set_device(dev)
+    if rank == 0:
+        _build.build_library()
+    if world > 1:
+        torch.distributed.barrier()
+    cfg = wl.CONFIGS[args.config]
+    if args.phys_layers:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
+    stream = torch.cuda.Stream()
+    total_steps = args.warmup + args.steps + (args.steps if not args.no_e2e else 0) + 1
+    t_setup = time.perf_counter()
+    with torch.cuda.stream(stream):
+        sess = DecodeSession(cfg, extra_tokens=total_steps + 1, device="cuda", stream=stream)
+        sess.fill_prefix()
+        L, B = cfg.num_layers, cfg.batch
+        qs, ks, vs = [], [], []
+        for l in range(L):
+            q, k, v = wl.step_inputs(cfg, 0, l, "cuda")
+            qs.append(q), ks.append(k), vs.append(v)
+        outs = [torch.empty_like(q) for q in qs]
+    stream.synchronize()
+    log(f"[rank {rank}] setup {time.perf_counter() - t_setup:.1f} s; pool "
+        f"{sess.query().pool_bytes / 2**30:.1f} GiB")
+
+    def step(events=None):
+        sess.begin_step()
+        for l in range(L):
+            sess.append(l, ks[l], vs[l])
+            if events is not None:
+                events[l][0].record(stream)
+            sess.attend(l, qs[l], outs[l])
+            if events is not None:
+                events[l][1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    stream.synchronize()
+
+    # ---- device-timed region
+    attended_per_step = []
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(L)]
+          for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_smi_id(torch, dev)) as clocks:
+        with torch.cuda.stream(stream):
+            start.record(stream)
+            for s in range(args.steps):
+                attended_per_step.append([int(n) + 1 for n in sess.lens])
+                step(ev[s])
+            stop.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    ms = start.elapsed_time(stop)
+    attn_ms = [e0.elapsed_time(e1) for evs in ev for (e0, e1) in evs]
+    step_bytes = []
+    attn_bytes = []
+    for att in attended_per_step:
+        a, p = layer_bytes(cfg, att)
+        step_bytes.append(L * (a + p))
+        attn_bytes.append(a)
+    st = sess.query()
+    assert st.device_error == 0, st.device_error
+
+    # ---- end to end: host inputs -> device -> host outputs, every step
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda t: t.cpu().pin_memory()
+        hq = [pin(q) for q in qs]
+        hk = [pin(k) for k in ks]
+        hv = [pin(v) for v in vs]
+        ho = [torch.empty_like(o, device="cpu").pin_memory() for o in outs]
+        dq = [torch.empty_like(q) for q in qs]
+        dk = [torch.empty_like(k) for k in ks]
+        dv = [torch.empty_like(v) for v in vs]
+        e_bytes = 0
+        h2d = sum(t.numel() * 2 for t in hq + hk + hv)
+        d2h = sum(t.numel() * 2 for t in ho)
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        w0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            s0.record(stream)
+            for s in range(args.steps):
+                att = [int(n) + 1 for n in sess.lens]
+                a, p = layer_bytes(cfg, att)
+                e_bytes += L * (a + p)
+                for l in range(L):
+                    dq[l].copy_(hq[l], non_blocking=True)
+                    dk[l].copy_(hk[l], non_blocking=True)
+                    dv[l].copy_(hv[l], non_blocking=True)
+                sess.begin_step()
+                for l in range(L):
+                    sess.append(l, dk[l], dv[l])
+                    sess.attend(l, dq[l], outs[l])
+                    ho[l].copy_(outs[l], non_blocking=True)
+            s1.record(stream)
+        stream.synchronize()
+        wall = time.perf_counter() - w0
+        e_ms = s0.elapsed_time(s1)
+        e2e = {"ms": e_ms, "wall_s": wall, "bytes": e_bytes, "h2d": h2d, "d2h": d2h}
+        st = sess.query()
+        assert st.device_error == 0
+
+    sess.close()
+    return {"ms": ms, "attn_ms": attn_ms, "step_bytes": step_bytes, "attn_bytes": attn_bytes,
+            "clocks": clocks.summary(), "e2e": e2e, "cfg": cfg, "L": L}
+
+
+def reduce_max(torch, x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="llava", choices=["tiny", "llava", "qwen", "ragged", "long"])
+    ap.add_argument("--phys-layers", type=int, default=0, help="layer pools held (profiling on a smaller cache)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget-s", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        log("warning: fewer than 3 warm-up steps")
+
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    from paper_2603_12707_gb300 import workloads as wl
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        cfg = wl.CONFIGS[args.config]
+        # each step: one layer of the workload through the float64 oracle
+        import torch
+        import oracle
+        lens = [int(n) + 1 for n in wl.context_lengths(cfg)]
+        k = torch.cat([wl.kv_block(cfg, 0, b, n, "k", "cpu") for b, n in enumerate(lens)])
+        v = torch.cat([wl.kv_block(cfg, 0, b, n, "v", "cpu") for b, n in enumerate(lens)])
+        q = wl.step_inputs(cfg, 0, 0, "cpu")[0]
+        for _ in range(args.warmup):
+            oracle.decode_attention(q, lens, k, v)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.decode_attention(q, lens, k, v)
+        dt = time.perf_counter() - t0
+        attn, _ = layer_bytes(cfg, lens)
+        val = attn * args.steps / dt / 1e9
+        threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+        sample = (f"per step: 1 of {cfg.num_layers} layers ({cfg.batch} sequences x {cfg.num_q_heads} heads) "
+                  f"of the {cfg.name} workload")
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": round(val, 4), "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": describe(cfg),
+            "cpu_baseline": {"value": round(val, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(val, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }))
+        return
+
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0))))
+    r = run_gpu(args, rank, world)
+    cfg, L = r["cfg"], r["L"]
+    ms = reduce_max(torch, r["ms"], world)
+    total_bytes = sum(r["step_bytes"]) * world
+    gbs = total_bytes / (ms / 1e3) / 1e9
+    steps_per_s = args.steps / (ms / 1e3)
+    attn_ms = statistics.mean(r["attn_ms"])
+    attn_bytes = statistics.mean(r["attn_bytes"])
+    peak, peak_kind = measured_peaks()
+    achieved = attn_bytes / (attn_ms / 1e3) / 1e9
+    traffic = committed_traffic(os.path.join(ROOT, "paper_2603_12707_gb300", "csrc", "kvd_decode.cu"))
+    out = {
+        "metric": METRIC, "value": round(gbs, 2), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {**describe(cfg), "l2": "each step streams the whole cache (far larger than the 129 MB L2)",
+                   "parallelism": f"replicas x{world}"},
+        "steps_per_s": round(steps_per_s * 1.0, 3),
+        "pct_of_measured_hbm": round(100 * gbs / world / peak, 2),
+        "pct_of_nominal_8tbs": round(100 * gbs / world / NOMINAL_HBM_GBS, 2),
+        "roofline": {"bound": "hbm", "kernel": "decode_attention", "achieved": round(achieved, 2),
+                     "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": (traffic["dram_bytes_per_launch_full"] if traffic else None),
+                     "algorithmic_bytes_per_launch": int(attn_bytes), "avg_launch_ms": round(attn_ms, 4)},
+        "clocks": r["clocks"],
+        "gpu_launches": args.steps * (1 + 2 * L),
+    }
+    if r["e2e"]:
+        e = r["e2e"]
+        e_ms = reduce_max(torch, e["ms"], world)
+        out["e2e"] = {"value": round(e["bytes"] * world / (e_ms / 1e3) / 1e9, 2), "unit": "GB/s",
+                      "h2d_bytes_per_step": e["h2d"], "d2h_bytes_per_step": e["d2h"],
+                      "steps_per_s": round(args.steps / (e_ms / 1e3), 3)}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        nbytes, secs, desc, threads = oracle_sample(cfg, args.cpu_budget_s)
+        out["cpu_baseline"] = {"value": round(nbytes / secs / 1e9, 4), "unit": "GB/s", "cores": threads,
+                               "kind": "oracle", "sample": desc}
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()

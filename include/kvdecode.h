@@ -1,0 +1,200 @@
+/*
+ * kvdecode.h -- C ABI of libkvdecode.so: paged bf16 KV cache and batched
+ * single-token decode attention for multimodal LLM serving on GB300 (sm_103a).
+ *
+ * The operation.  Language decoding is the memory-bandwidth-bound phase of
+ * multimodal inference: every step streams the KV cache from HBM
+ * (HeteroServe, Sec. 2 "Language decoding"; Sec. 5.1 datacenter pool running
+ * decode with MHA and GQA backends).  The cache of one request holds
+ * s_ctx = N_v + s_text tokens for each of L layers and n_kv KV heads of
+ * dimension d_h, 2 * L * n_kv * d_h * s_ctx * b bytes (Sec. 4.1, Eq. 1), and
+ * its first N_v positions are the KV of the vision embedding handed over at
+ * the modality boundary (Sec. 5.1, the [1, N_v, d] embedding).  Blocks of the
+ * cache are taken lazily, only when a request needs them (Sec. 5.4 "Lazy KV
+ * Cache Allocation").  One decode step of one layer computes, for sequence b,
+ * query head h and KV head g = h / G (G = H_q / H_kv):
+ *
+ *     o[b][h] = sum_t softmax_t(scale * q[b][h] . k[b][g][t]) * v[b][g][t]
+ *
+ * over all cached tokens t of b in logical order, including the token that
+ * kv_append wrote for this step.
+ *
+ * Conventions for every function below.
+ *  - Return KVC_OK (0) or a negative KVC_ERR_* code; kv_last_error() then
+ *    returns a message for the calling thread.  On error nothing has been
+ *    changed and nothing has been enqueued, unless the description says so.
+ *  - bf16 tensors are IEEE bfloat16 bit patterns, row-major, densely packed.
+ *  - "device" pointers must be CUDA device (or managed) memory of the device
+ *    that was current at kv_cache_create; "host" pointers are ordinary host
+ *    memory that the call reads before returning.  The caller owns every
+ *    pointer it passes; the cache owns its pools, page table and scratch.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Device work
+ *    is enqueued on it asynchronously; no hot-path call synchronises.  All
+ *    calls on one cache must be ordered on one stream (or externally
+ *    synchronised): the cache's scratch is shared between calls.
+ *  - A handle must not be used from two host threads at once.
+ */
+#ifndef KVDECODE_H
+#define KVDECODE_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KVC_API __attribute__((visibility("default")))
+#else
+#define KVC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define KVC_OK 0
+#define KVC_ERR_INVALID (-1)      /* bad argument, shape or sequence id      */
+#define KVC_ERR_OOM (-2)          /* page pool or device memory exhausted     */
+#define KVC_ERR_CUDA (-3)         /* a CUDA runtime call failed               */
+#define KVC_ERR_PAGE_TABLE (-4)   /* device found a page id outside the pool  */
+#define KVC_ERR_UNSUPPORTED (-5)  /* valid but unsupported shape              */
+#define KVC_ERR_DEVICE (-6)       /* device-side wait gave up (see stats)     */
+
+/* kvc_config.flags */
+#define KVC_FLAG_HOST_ONLY 1  /* bookkeeping only: no device memory, no kernels.
+                                 Allocation, page tables and sequence calls work;
+                                 data and attention calls return KVC_ERR_INVALID. */
+
+/* kvc_stats.device_error bits (sticky until the cache is destroyed) */
+#define KVC_DEVERR_PAGE_RANGE 1   /* a page-table entry outside [0, num_pages) */
+#define KVC_DEVERR_WAIT_TIMEOUT 2 /* a shared-memory pipeline wait gave up      */
+#define KVC_DEVERR_SEQ_RANGE 4    /* a sequence length outside its page row     */
+
+typedef struct kvc_config {
+    int32_t num_layers;        /* L: layer pools held (>= 1)                              */
+    int32_t num_q_heads;       /* H_q (multiple of num_kv_heads)                          */
+    int32_t num_kv_heads;      /* H_kv; G = H_q / H_kv must be <= 8                       */
+    int32_t head_dim;          /* d_h: 64 or 128                                          */
+    int32_t page_size;         /* P: tokens per page; 16                                  */
+    int32_t max_seqs;          /* sequence slots (ids 0 .. max_seqs-1), <= 65535          */
+    int32_t max_pages_per_seq; /* page-table row length                                   */
+    int32_t flags;             /* KVC_FLAG_*                                              */
+    int64_t num_pages;         /* pages in the pool; one page id addresses the same slot
+                                  in every layer pool, for K and for V                    */
+} kvc_config;
+
+typedef struct kvc_stats {
+    int64_t kv_bytes_allocated; /* bytes of the pages in use: Eq. 1 with s_ctx rounded up
+                                   to whole pages, 2 * L * H_kv * d_h * 2 * P * pages_in_use */
+    int64_t pool_bytes;         /* bytes of the K and V pools on the device              */
+    int64_t pages_in_use;
+    int64_t free_pages;
+    int32_t live_seqs;
+    int32_t device_error;       /* KVC_DEVERR_* bits found by kernels so far             */
+} kvc_stats;
+
+typedef struct kv_cache kv_cache; /* opaque */
+
+/* ---------------------------------------------------------------- cache -- */
+
+/* Create a cache on the current CUDA device.  Allocates the K and V pools,
+ * each laid out [L][num_pages][H_kv][P][d_h] bf16 (one (page, head) tile is
+ * P * d_h * 2 bytes of consecutive tokens), the page table
+ * [max_seqs][max_pages_per_seq] int32 (unused entries -1), the lengths, and
+ * step scratch; zero-fills the pools on `stream`.  Initial page pop order is
+ * 0, 1, 2, ...  KVC_ERR_UNSUPPORTED for head_dim not in {64, 128},
+ * page_size != 16 or G > 8; KVC_ERR_OOM if device memory runs out. */
+KVC_API int kv_cache_create(const kvc_config *cfg, void *stream, kv_cache **out);
+
+/* Free everything the cache owns (stream-ordered on the creation stream,
+ * after a device synchronisation of that stream).  NULL is accepted. */
+KVC_API int kv_cache_destroy(kv_cache *cache);
+
+/* Install the order in which free pages are handed out: order[0] first.
+ * `order` (host, n = num_pages entries) must be a permutation of
+ * 0 .. num_pages-1, and no page may be in use. */
+KVC_API int kv_cache_set_page_order(kv_cache *cache, const int32_t *order, int64_t n);
+
+/* Synchronise the cache's stream and report usage and device error bits.
+ * Returns KVC_ERR_PAGE_TABLE / KVC_ERR_DEVICE if device_error is non-zero
+ * (the stats are filled in either way). */
+KVC_API int kv_cache_query(kv_cache *cache, kvc_stats *stats);
+
+/* Device pointers of one layer's K and V pools ([num_pages][H_kv][P][d_h]
+ * bf16), for inspection; owned by the cache. */
+KVC_API int kv_cache_pool(kv_cache *cache, int32_t layer, void **k_pool, void **v_pool);
+
+/* Override the split size (pages per work item of decode_attention) used
+ * by later kv_begin_step calls; 0 restores the automatic choice.
+ * Range 0 .. 64. */
+KVC_API int kv_cache_set_split_pages(kv_cache *cache, int32_t pages);
+
+/* -------------------------------------------------------- sequences ------ */
+
+/* Open a sequence of length 0; *seq_id = the lowest free id.  No page is
+ * taken until tokens are reserved (lazy allocation, Sec. 5.4). */
+KVC_API int kv_seq_create(kv_cache *cache, int32_t *seq_id);
+
+/* Reserve n_tokens more positions at the end of a sequence.  Walking the new
+ * positions in order, a page is taken from the pop order exactly when a
+ * position is the first slot of a page.  All or nothing: KVC_ERR_OOM if the
+ * pool lacks pages, KVC_ERR_INVALID if the row would exceed
+ * max_pages_per_seq.  The page-table and length update is enqueued on
+ * `stream`. */
+KVC_API int kv_seq_reserve(kv_cache *cache, int32_t seq_id, int32_t n_tokens, void *stream);
+
+/* Close a sequence: its pages go back to the front of the pop order in its
+ * logical page order.  The device row is reset on `stream`. */
+KVC_API int kv_seq_free(kv_cache *cache, int32_t seq_id, void *stream);
+
+/* Host view of one sequence: *len = reserved positions; page_ids (host,
+ * capacity entries, may be NULL) receives its pages in logical order;
+ * *n_pages = ceil(len / P). */
+KVC_API int kv_seq_info(kv_cache *cache, int32_t seq_id, int32_t *len, int32_t *page_ids,
+                int32_t capacity, int32_t *n_pages);
+
+/* Write n tokens of one layer into reserved positions [first_pos,
+ * first_pos + n) of a sequence: the prefix (the N_v vision tokens handed over
+ * at the modality boundary, then the prompt) or any later rewrite.
+ * k, v: device, [n][H_kv][d_h] bf16.  Requires first_pos + n <= length. */
+KVC_API int kv_write_tokens(kv_cache *cache, int32_t layer, int32_t seq_id, int32_t first_pos,
+                    int32_t n, const void *k, const void *v, void *stream);
+
+/* Copy positions [first_pos, first_pos + n) of one layer back into logical
+ * order: k_out, v_out device [n][H_kv][d_h] bf16. */
+KVC_API int kv_read_tokens(kv_cache *cache, int32_t layer, int32_t seq_id, int32_t first_pos,
+                   int32_t n, void *k_out, void *v_out, void *stream);
+
+/* -------------------------------------------------------- decode step ---- */
+
+/* Start one decode step for `batch` distinct live sequences (seq_ids: host,
+ * batch entries; batch order is the row order of q, out, k_new, v_new in the
+ * calls below).  Reserves one position s_b (the old length) per sequence,
+ * taking a page when s_b % P == 0, all or nothing (KVC_ERR_OOM leaves
+ * everything unchanged), and enqueues one kernel that updates the device page
+ * table and lengths and builds the split plan the layers of this step share.
+ * batch <= max_seqs. */
+KVC_API int kv_begin_step(kv_cache *cache, int32_t batch, const int32_t *seq_ids, void *stream);
+
+/* Fused K+V append for one layer of the current step: writes k_new[b] and
+ * v_new[b] (device, [batch][H_kv][d_h] bf16) into position s_b of each
+ * sequence of the step.  `batch` must equal the step's batch. */
+KVC_API int kv_append(kv_cache *cache, int32_t layer, int32_t batch, const void *k_new,
+              const void *v_new, void *stream);
+
+/* Decode attention for one layer of the current step.  q: device
+ * [batch][H_q][d_h] bf16; out: device [batch][H_q][d_h] bf16 (written).
+ * Attends over positions 0 .. s_b of each sequence, so call kv_append for the
+ * same layer first, on the same stream.  softmax_scale <= 0 selects
+ * 1/sqrt(d_h).  Split-KV: the step's plan cuts each (sequence, KV head) into
+ * work items of consecutive pages; each item runs an online softmax in fp32
+ * over its pages for all G query heads of the KV head, and the last item of a
+ * (sequence, KV head) to finish merges the partial results by log-sum-exp. */
+KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, const void *q, void *out,
+                     float softmax_scale, void *stream);
+
+/* Message of the last failed call on this thread ("" if none). */
+KVC_API const char *kv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVDECODE_H */

@@ -1,0 +1,191 @@
+// Page-table maintenance, the per-step update and split plan, token writes /
+// reads into pages, and the fused K+V append (kv_append).
+#include "kvd_internal.h"
+
+namespace kvd {
+
+namespace {
+
+__device__ __forceinline__ void flag_error(int32_t* err, int bit) { atomicOr(err, bit); }
+
+__global__ void scatter_i32_kernel(int32_t* base, const __grid_constant__ ScatterI32 s)
+{
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < s.n; i += gridDim.x * blockDim.x)
+        base[s.idx[i]] = s.val[i];
+}
+
+// Exclusive block-wide prefix sum of one int per thread (blockDim.x = 1024).
+__device__ int block_exclusive_scan(int v, int* total)
+{
+    __shared__ int warp_sums[32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = (lane < (int)(blockDim.x >> 5)) ? warp_sums[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        warp_sums[lane] = w;   // inclusive over warps
+    }
+    __syncthreads();
+    const int before_warp = warp ? warp_sums[warp - 1] : 0;
+    *total = warp_sums[31];
+    __syncthreads();
+    return before_warp + x - v;
+}
+
+// Apply the step's length / page-table updates; in the last launch of a step,
+// build the split plan: each batch row's pages cut into items of C pages,
+// full items first (in row order), then every row's shorter last item.
+__global__ void __launch_bounds__(1024)
+    step_kernel(const __grid_constant__ StepPatch patch, const PlanArgs a, int32_t total_full)
+{
+    for (int i = threadIdx.x; i < patch.n; i += blockDim.x) {
+        const int seq = patch.seq[i], len = patch.new_len[i];
+        a.seq_len[seq] = len;
+        a.step_seq[patch.b0 + i] = seq;
+        if (patch.new_page[i] >= 0)
+            a.page_table[(int64_t)seq * a.max_pages + (len - 1) / kPageSize] = patch.new_page[i];
+    }
+    if (!a.build) return;
+    __syncthreads();
+    const int C = a.chunk_pages;
+    int carry_full = 0, carry_rem = 0, carry_nch = 0;
+    for (int base = 0; base < a.batch; base += blockDim.x) {
+        const int b = base + threadIdx.x;
+        int seq = 0, len = 0, np = 0;
+        if (b < a.batch) {
+            seq = a.step_seq[b];
+            len = a.seq_len[seq];
+            if (len <= 0 || len > a.max_pages * kPageSize) {
+                flag_error(a.err, 4);
+                len = 1;
+            }
+            np = (len + kPageSize - 1) / kPageSize;
+        }
+        const int full = np / C, rem = (np % C) ? 1 : 0, nch = full + rem;
+        int t_full, t_rem, t_nch;
+        const int ex_full = block_exclusive_scan(full, &t_full);
+        const int ex_rem = block_exclusive_scan(rem, &t_rem);
+        const int ex_nch = block_exclusive_scan(nch, &t_nch);
+        if (b < a.batch) {
+            const int slot_base = carry_nch + ex_nch;
+            for (int c = 0; c < full; ++c) {
+                PlanEntry e{b, seq, len, c * C, C, c, nch, slot_base};
+                a.plan[carry_full + ex_full + c] = e;
+            }
+            if (rem) {
+                PlanEntry e{b, seq, len, full * C, np - full * C, full, nch, slot_base};
+                a.plan[total_full + carry_rem + ex_rem] = e;
+            }
+        }
+        carry_full += t_full;
+        carry_rem += t_rem;
+        carry_nch += t_nch;
+    }
+}
+
+// One thread per 16-byte chunk of a [n][H_kv][D] token block.
+__global__ void token_copy_kernel(const TokenCopyArgs a)
+{
+    const int chunks = a.D / 8;
+    const int64_t total = (int64_t)a.n * a.H_kv * chunks;
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % chunks);
+        const int64_t tg = i / chunks;
+        const int g = (int)(tg % a.H_kv);
+        const int t = (int)(tg / a.H_kv);
+        const int pos = a.first_pos + t;
+        const int32_t page = a.pt_row[pos / kPageSize];
+        if (page < 0 || page >= a.num_pages) {
+            flag_error(a.err, 1);
+            continue;
+        }
+        const int64_t poff = (((int64_t)page * a.H_kv + g) * kPageSize + pos % kPageSize) * a.D + c * 8;
+        const int64_t toff = i * 8;
+        if (a.to_pool) {
+            *reinterpret_cast<uint4*>(a.pool_k + poff) = *reinterpret_cast<const uint4*>(a.tok_k + toff);
+            *reinterpret_cast<uint4*>(a.pool_v + poff) = *reinterpret_cast<const uint4*>(a.tok_v + toff);
+        } else {
+            *reinterpret_cast<uint4*>(a.tok_k + toff) = *reinterpret_cast<const uint4*>(a.pool_k + poff);
+            *reinterpret_cast<uint4*>(a.tok_v + toff) = *reinterpret_cast<const uint4*>(a.pool_v + poff);
+        }
+    }
+}
+
+// kv_append: one thread per 16-byte chunk of k_new / v_new ([B][H_kv][D]);
+// the chunk goes to slot (len-1) % P of page page_table[seq][(len-1) / P].
+__global__ void append_kernel(const AppendArgs a)
+{
+    const int chunks = a.D / 8;
+    const int total = a.batch * a.H_kv * chunks;
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= total) return;
+    const int c = i % chunks;
+    const int bg = i / chunks;
+    const int g = bg % a.H_kv;
+    const int b = bg / a.H_kv;
+    const int seq = a.step_seq[b];
+    const int pos = a.seq_len[seq] - 1;
+    if (pos < 0 || pos >= a.max_pages * kPageSize) {
+        flag_error(a.err, 4);
+        return;
+    }
+    const int32_t page = a.page_table[(int64_t)seq * a.max_pages + pos / kPageSize];
+    if (page < 0 || page >= a.num_pages) {
+        flag_error(a.err, 1);
+        return;
+    }
+    const int64_t poff = (((int64_t)page * a.H_kv + g) * kPageSize + pos % kPageSize) * a.D + c * 8;
+    const int64_t noff = (int64_t)i * 8;
+    const uint4 kk = *reinterpret_cast<const uint4*>(a.k_new + noff);
+    const uint4 vv = *reinterpret_cast<const uint4*>(a.v_new + noff);
+    *reinterpret_cast<uint4*>(a.pool_k + poff) = kk;
+    *reinterpret_cast<uint4*>(a.pool_v + poff) = vv;
+}
+
+}  // namespace
+
+cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st)
+{
+    if (s.n <= 0) return cudaSuccess;
+    scatter_i32_kernel<<<(s.n + 255) / 256, 256, 0, st>>>(base, s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, int32_t total_full,
+                        cudaStream_t st)
+{
+    step_kernel<<<1, 1024, 0, st>>>(patch, plan, total_full);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st)
+{
+    const int64_t total = (int64_t)a.n * a.H_kv * (a.D / 8);
+    if (total <= 0) return cudaSuccess;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 65535) blocks = 65535;
+    token_copy_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t st)
+{
+    const int total = a.batch * a.H_kv * (a.D / 8);
+    if (total <= 0) return cudaSuccess;
+    append_kernel<<<(total + 255) / 256, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace kvd

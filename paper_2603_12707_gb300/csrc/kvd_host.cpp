@@ -1,0 +1,613 @@
+// Host side of libkvdecode.so: the C ABI, argument checking, the lazy page
+// allocator with its host mirror of the page table, the per-step split plan
+// sizing, TMA descriptors, and kernel launches.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "kvd_internal.h"
+#include "kvdecode.h"
+
+using namespace kvd;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const std::string& msg)
+{
+    g_last_error = msg;
+    return code;
+}
+
+#define KVD_CUDA(call)                                                                       \
+    do {                                                                                     \
+        cudaError_t e_ = (call);                                                             \
+        if (e_ != cudaSuccess)                                                               \
+            return fail(e_ == cudaErrorMemoryAllocation ? KVC_ERR_OOM : KVC_ERR_CUDA,        \
+                        std::string(#call) + ": " + cudaGetErrorString(e_));                 \
+    } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+struct kv_cache {
+    kvc_config cfg{};
+    bool host_only = false;
+    int device = 0;
+    int group = 1;
+    int num_sms = 0;
+    DecodeVariant variant{};
+
+    // host allocator state
+    std::vector<int32_t> free_stack;            // back() is handed out next
+    std::vector<int32_t> lens;                  // -1: sequence id not in use
+    std::vector<std::vector<int32_t>> pages;    // logical page -> physical page
+    int64_t pages_in_use = 0;
+    int32_t live = 0;
+    std::vector<uint32_t> stamp;                // duplicate check in kv_begin_step
+    uint32_t stamp_gen = 0;
+
+    // device memory
+    uint16_t* pools = nullptr;                  // [2][L][num_pages][H_kv][P][D]
+    size_t layer_elems = 0;
+    int32_t* meta = nullptr;                    // page table [max_seqs][max_pages], then seq_len [max_seqs]
+    int32_t* step_seq = nullptr;
+    int32_t* tickets = nullptr;
+    uint32_t* queue = nullptr;
+    int32_t* err = nullptr;
+    PlanEntry* plan = nullptr;
+    int64_t plan_cap = 0;
+    float* part_o = nullptr;
+    float2* part_ml = nullptr;
+    int64_t slot_cap = 0;
+    std::vector<CUtensorMap> tmaps;             // [L][2]: K, V
+
+    // current step
+    bool step_active = false;
+    int32_t step_batch = 0;
+    int32_t step_entries = 0;
+    int32_t split_override = 0;
+
+    int32_t* page_table() const { return meta; }
+    int32_t* seq_len_dev() const { return meta + (int64_t)cfg.max_seqs * cfg.max_pages_per_seq; }
+    int32_t seq_len_index(int32_t seq) const { return cfg.max_seqs * cfg.max_pages_per_seq + seq; }
+    uint16_t* k_pool(int layer) const { return pools + (size_t)layer * layer_elems; }
+    uint16_t* v_pool(int layer) const { return pools + ((size_t)cfg.num_layers + layer) * layer_elems; }
+
+    int32_t pop_page()
+    {
+        const int32_t p = free_stack.back();
+        free_stack.pop_back();
+        ++pages_in_use;
+        return p;
+    }
+};
+
+namespace {
+
+int check_seq(const kv_cache* c, int32_t seq)
+{
+    if (seq < 0 || seq >= c->cfg.max_seqs || c->lens[seq] < 0)
+        return fail(KVC_ERR_INVALID, "sequence id " + std::to_string(seq) + " is not live");
+    return KVC_OK;
+}
+
+int check_device(const kv_cache* c, const char* what)
+{
+    if (c->host_only) return fail(KVC_ERR_INVALID, std::string(what) + ": cache was created host-only");
+    return KVC_OK;
+}
+
+// Enqueue int32 updates of the page table / lengths.
+int push_updates(kv_cache* c, const std::vector<int32_t>& idx, const std::vector<int32_t>& val,
+                 cudaStream_t st)
+{
+    if (c->host_only || idx.empty()) return KVC_OK;
+    ScatterI32 s;
+    for (size_t off = 0; off < idx.size(); off += kScatterMax) {
+        const size_t n = std::min<size_t>(kScatterMax, idx.size() - off);
+        s.n = (int32_t)n;
+        std::memcpy(s.idx, idx.data() + off, n * sizeof(int32_t));
+        std::memcpy(s.val, val.data() + off, n * sizeof(int32_t));
+        KVD_CUDA(launch_scatter_i32(c->meta, s, st));
+    }
+    return KVC_OK;
+}
+
+int32_t auto_split_pages(const kv_cache* c, int64_t total_units)
+{
+    // Aim for about four work items per resident warp so the tail of the
+    // persistent schedule stays short, within [2, kMaxSplitPages] pages.
+    const int64_t warps = (int64_t)std::max(1, c->num_sms) * std::max(1, c->variant.ctas_per_sm) *
+                          std::max(1, c->variant.warps);
+    int64_t C = (total_units + 4 * warps - 1) / (4 * warps);
+    return (int32_t)std::min<int64_t>(kMaxSplitPages, std::max<int64_t>(2, C));
+}
+
+int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, cudaStream_t st)
+{
+    if (entries > c->plan_cap) {
+        const int64_t cap = std::max<int64_t>(entries, c->plan_cap + c->plan_cap / 2);
+        if (c->plan) KVD_CUDA(cudaFreeAsync(c->plan, st));
+        c->plan = nullptr;
+        c->plan_cap = 0;
+        KVD_CUDA(cudaMallocAsync((void**)&c->plan, (size_t)cap * sizeof(PlanEntry), st));
+        c->plan_cap = cap;
+    }
+    if (slots > c->slot_cap) {
+        const int64_t cap = std::max<int64_t>(slots, c->slot_cap + c->slot_cap / 2);
+        if (c->part_o) KVD_CUDA(cudaFreeAsync(c->part_o, st));
+        if (c->part_ml) KVD_CUDA(cudaFreeAsync(c->part_ml, st));
+        c->part_o = nullptr;
+        c->part_ml = nullptr;
+        c->slot_cap = 0;
+        const size_t G = (size_t)c->group, D = (size_t)c->cfg.head_dim;
+        KVD_CUDA(cudaMallocAsync((void**)&c->part_o, (size_t)cap * G * D * sizeof(float), st));
+        KVD_CUDA(cudaMallocAsync((void**)&c->part_ml, (size_t)cap * G * sizeof(float2), st));
+        c->slot_cap = cap;
+    }
+    return KVC_OK;
+}
+
+void release_device(kv_cache* c)
+{
+    cudaFree(c->pools);
+    cudaFree(c->meta);
+    cudaFree(c->step_seq);
+    cudaFree(c->tickets);
+    cudaFree(c->queue);
+    cudaFree(c->err);
+    cudaFree(c->plan);
+    cudaFree(c->part_o);
+    cudaFree(c->part_ml);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* kv_last_error(void) { return g_last_error.c_str(); }
+
+int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
+{
+    if (!cfg || !out) return fail(KVC_ERR_INVALID, "kv_cache_create: null argument");
+    *out = nullptr;
+    const kvc_config& k = *cfg;
+    if (k.num_layers < 1 || k.num_q_heads < 1 || k.num_kv_heads < 1 || k.head_dim < 1 ||
+        k.page_size < 1 || k.max_seqs < 1 || k.max_pages_per_seq < 1 || k.num_pages < 1)
+        return fail(KVC_ERR_INVALID, "kv_cache_create: every size must be positive");
+    if (k.num_q_heads % k.num_kv_heads != 0)
+        return fail(KVC_ERR_INVALID, "kv_cache_create: num_q_heads must be a multiple of num_kv_heads");
+    if (k.num_q_heads / k.num_kv_heads > kMaxGroup)
+        return fail(KVC_ERR_UNSUPPORTED, "kv_cache_create: more than 8 query heads per KV head");
+    if (k.head_dim != 64 && k.head_dim != 128)
+        return fail(KVC_ERR_UNSUPPORTED, "kv_cache_create: head_dim must be 64 or 128");
+    if (k.page_size != kPageSize) return fail(KVC_ERR_UNSUPPORTED, "kv_cache_create: page_size must be 16");
+    if (k.max_seqs > 65535) return fail(KVC_ERR_INVALID, "kv_cache_create: max_seqs > 65535");
+    if ((int64_t)k.max_seqs * k.max_pages_per_seq + k.max_seqs >= (int64_t)1 << 31)
+        return fail(KVC_ERR_INVALID, "kv_cache_create: page table larger than 2^31 entries");
+    if (k.num_pages * k.num_kv_heads * kPageSize >= (int64_t)1 << 31)
+        return fail(KVC_ERR_INVALID, "kv_cache_create: num_pages * num_kv_heads * 16 must be < 2^31");
+    if (k.flags & ~KVC_FLAG_HOST_ONLY) return fail(KVC_ERR_INVALID, "kv_cache_create: unknown flag");
+
+    kv_cache* c = new kv_cache();
+    c->cfg = k;
+    c->host_only = (k.flags & KVC_FLAG_HOST_ONLY) != 0;
+    c->group = k.num_q_heads / k.num_kv_heads;
+    c->lens.assign(k.max_seqs, -1);
+    c->pages.assign(k.max_seqs, {});
+    c->stamp.assign(k.max_seqs, 0);
+    c->free_stack.resize(k.num_pages);
+    for (int64_t i = 0; i < k.num_pages; ++i) c->free_stack[i] = (int32_t)(k.num_pages - 1 - i);
+
+    if (!c->host_only) {
+        cudaStream_t st = static_cast<cudaStream_t>(stream);
+        auto bail = [&](int rc) {
+            release_device(c);
+            delete c;
+            return rc;
+        };
+#define KVD_CUDA_C(call)                                                                    \
+    do {                                                                                    \
+        cudaError_t e_ = (call);                                                            \
+        if (e_ != cudaSuccess)                                                              \
+            return bail(fail(e_ == cudaErrorMemoryAllocation ? KVC_ERR_OOM : KVC_ERR_CUDA,  \
+                             std::string(#call) + ": " + cudaGetErrorString(e_)));         \
+    } while (0)
+        KVD_CUDA_C(cudaGetDevice(&c->device));
+        KVD_CUDA_C(cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device));
+        KVD_CUDA_C(decode_variant_info(k.head_dim, c->group > 1, &c->variant));
+        auto encode = tensor_map_encoder();
+        if (!encode) return bail(fail(KVC_ERR_CUDA, "kv_cache_create: cuTensorMapEncodeTiled unavailable"));
+
+        c->layer_elems = (size_t)k.num_pages * k.num_kv_heads * kPageSize * k.head_dim;
+        const size_t pool_bytes = 2 * (size_t)k.num_layers * c->layer_elems * sizeof(uint16_t);
+        const size_t meta_elems = (size_t)k.max_seqs * k.max_pages_per_seq + k.max_seqs;
+        KVD_CUDA_C(cudaMalloc((void**)&c->pools, pool_bytes));
+        KVD_CUDA_C(cudaMalloc((void**)&c->meta, meta_elems * sizeof(int32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->step_seq, (size_t)k.max_seqs * sizeof(int32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->tickets, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->queue, 2 * sizeof(uint32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->err, sizeof(int32_t)));
+        KVD_CUDA_C(cudaMemsetAsync(c->pools, 0, pool_bytes, st));
+        KVD_CUDA_C(cudaMemsetAsync(c->meta, 0xff, (size_t)k.max_seqs * k.max_pages_per_seq * sizeof(int32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->seq_len_dev(), 0, (size_t)k.max_seqs * sizeof(int32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->step_seq, 0, (size_t)k.max_seqs * sizeof(int32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->tickets, 0, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->queue, 0, 2 * sizeof(uint32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->err, 0, sizeof(int32_t), st));
+#undef KVD_CUDA_C
+
+        // One 2-D view per layer pool: rows = (page * H_kv + head) * P + slot,
+        // D bf16 columns; tiles are boxes of 16 rows x 64 columns, 128-byte swizzle.
+        c->tmaps.resize(2 * (size_t)k.num_layers);
+        for (int l = 0; l < k.num_layers; ++l) {
+            for (int kv = 0; kv < 2; ++kv) {
+                void* base = kv ? c->v_pool(l) : c->k_pool(l);
+                cuuint64_t gdim[2] = {(cuuint64_t)k.head_dim, (cuuint64_t)(k.num_pages * k.num_kv_heads * kPageSize)};
+                cuuint64_t gstride[1] = {(cuuint64_t)k.head_dim * sizeof(uint16_t)};
+                cuuint32_t box[2] = {64, (cuuint32_t)kPageSize};
+                cuuint32_t estride[2] = {1, 1};
+                CUresult r = encode(&c->tmaps[2 * l + kv], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, gdim, gstride,
+                                    box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                if (r != CUDA_SUCCESS) {
+                    release_device(c);
+                    delete c;
+                    return fail(KVC_ERR_CUDA, "kv_cache_create: cuTensorMapEncodeTiled failed (" +
+                                                  std::to_string((int)r) + ")");
+                }
+            }
+        }
+    }
+    *out = c;
+    return KVC_OK;
+}
+
+int kv_cache_destroy(kv_cache* c)
+{
+    if (!c) return KVC_OK;
+    int rc = KVC_OK;
+    if (!c->host_only) {
+        cudaError_t e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) rc = fail(KVC_ERR_CUDA, std::string("kv_cache_destroy: ") + cudaGetErrorString(e));
+        release_device(c);
+    }
+    delete c;
+    return rc;
+}
+
+int kv_cache_set_page_order(kv_cache* c, const int32_t* order, int64_t n)
+{
+    if (!c || !order) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: null argument");
+    if (n != c->cfg.num_pages) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: n must equal num_pages");
+    if (c->pages_in_use) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: pages are in use");
+    std::vector<uint8_t> seen((size_t)n, 0);
+    for (int64_t i = 0; i < n; ++i) {
+        if (order[i] < 0 || order[i] >= n || seen[order[i]])
+            return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: not a permutation of the pool");
+        seen[order[i]] = 1;
+    }
+    for (int64_t i = 0; i < n; ++i) c->free_stack[i] = order[n - 1 - i];
+    return KVC_OK;
+}
+
+int kv_cache_query(kv_cache* c, kvc_stats* s)
+{
+    if (!c || !s) return fail(KVC_ERR_INVALID, "kv_cache_query: null argument");
+    const kvc_config& k = c->cfg;
+    s->pages_in_use = c->pages_in_use;
+    s->free_pages = (int64_t)c->free_stack.size();
+    s->kv_bytes_allocated = 2 * (int64_t)k.num_layers * k.num_kv_heads * k.head_dim * 2 * kPageSize * c->pages_in_use;
+    s->pool_bytes = c->host_only ? 0 : (int64_t)(2 * (size_t)k.num_layers * c->layer_elems * sizeof(uint16_t));
+    s->live_seqs = c->live;
+    s->device_error = 0;
+    if (c->host_only) return KVC_OK;
+    KVD_CUDA(cudaDeviceSynchronize());
+    KVD_CUDA(cudaMemcpy(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost));
+    if (s->device_error & (KVC_DEVERR_PAGE_RANGE | KVC_DEVERR_SEQ_RANGE))
+        return fail(KVC_ERR_PAGE_TABLE, "device found a page id or length outside its range");
+    if (s->device_error) return fail(KVC_ERR_DEVICE, "a device-side pipeline wait gave up");
+    return KVC_OK;
+}
+
+int kv_cache_pool(kv_cache* c, int32_t layer, void** k_pool, void** v_pool)
+{
+    if (!c || !k_pool || !v_pool) return fail(KVC_ERR_INVALID, "kv_cache_pool: null argument");
+    if (int rc = check_device(c, "kv_cache_pool")) return rc;
+    if (layer < 0 || layer >= c->cfg.num_layers) return fail(KVC_ERR_INVALID, "kv_cache_pool: bad layer");
+    *k_pool = c->k_pool(layer);
+    *v_pool = c->v_pool(layer);
+    return KVC_OK;
+}
+
+int kv_cache_set_split_pages(kv_cache* c, int32_t pages)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_cache_set_split_pages: null cache");
+    if (pages < 0 || pages > kMaxSplitPages)
+        return fail(KVC_ERR_INVALID, "kv_cache_set_split_pages: pages must be in 0 .. 64");
+    c->split_override = pages;
+    return KVC_OK;
+}
+
+int kv_seq_create(kv_cache* c, int32_t* seq_id)
+{
+    if (!c || !seq_id) return fail(KVC_ERR_INVALID, "kv_seq_create: null argument");
+    for (int32_t i = 0; i < c->cfg.max_seqs; ++i) {
+        if (c->lens[i] < 0) {
+            c->lens[i] = 0;
+            c->pages[i].clear();
+            ++c->live;
+            *seq_id = i;
+            return KVC_OK;
+        }
+    }
+    return fail(KVC_ERR_OOM, "kv_seq_create: every sequence slot is in use");
+}
+
+int kv_seq_reserve(kv_cache* c, int32_t seq, int32_t n, void* stream)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_seq_reserve: null cache");
+    if (int rc = check_seq(c, seq)) return rc;
+    if (n < 0) return fail(KVC_ERR_INVALID, "kv_seq_reserve: negative token count");
+    const int64_t len = c->lens[seq], new_len = len + n;
+    const int64_t have = (len + kPageSize - 1) / kPageSize, need = (new_len + kPageSize - 1) / kPageSize;
+    if (need > c->cfg.max_pages_per_seq) return fail(KVC_ERR_INVALID, "kv_seq_reserve: page-table row too short");
+    if (need - have > (int64_t)c->free_stack.size()) return fail(KVC_ERR_OOM, "kv_seq_reserve: page pool exhausted");
+    if (n == 0) return KVC_OK;
+    std::vector<int32_t> idx, val;
+    for (int64_t p = have; p < need; ++p) {
+        const int32_t page = c->pop_page();
+        c->pages[seq].push_back(page);
+        idx.push_back(seq * c->cfg.max_pages_per_seq + (int32_t)p);
+        val.push_back(page);
+    }
+    c->lens[seq] = (int32_t)new_len;
+    idx.push_back(c->seq_len_index(seq));
+    val.push_back((int32_t)new_len);
+    return push_updates(c, idx, val, static_cast<cudaStream_t>(stream));
+}
+
+int kv_seq_free(kv_cache* c, int32_t seq, void* stream)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_seq_free: null cache");
+    if (int rc = check_seq(c, seq)) return rc;
+    std::vector<int32_t> idx, val;
+    auto& pg = c->pages[seq];
+    for (size_t i = 0; i < pg.size(); ++i) {
+        idx.push_back(seq * c->cfg.max_pages_per_seq + (int32_t)i);
+        val.push_back(-1);
+    }
+    for (size_t i = pg.size(); i-- > 0;) c->free_stack.push_back(pg[i]);
+    c->pages_in_use -= (int64_t)pg.size();
+    pg.clear();
+    c->lens[seq] = -1;
+    --c->live;
+    c->step_active = false;
+    idx.push_back(c->seq_len_index(seq));
+    val.push_back(0);
+    return push_updates(c, idx, val, static_cast<cudaStream_t>(stream));
+}
+
+int kv_seq_info(kv_cache* c, int32_t seq, int32_t* len, int32_t* page_ids, int32_t capacity, int32_t* n_pages)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_seq_info: null cache");
+    if (int rc = check_seq(c, seq)) return rc;
+    const auto& pg = c->pages[seq];
+    if (len) *len = c->lens[seq];
+    if (n_pages) *n_pages = (int32_t)pg.size();
+    if (page_ids)
+        for (int32_t i = 0; i < capacity && i < (int32_t)pg.size(); ++i) page_ids[i] = pg[i];
+    return KVC_OK;
+}
+
+static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq, int32_t first, int32_t n,
+                      void* k, void* v, int to_pool, void* stream)
+{
+    if (!c) return fail(KVC_ERR_INVALID, std::string(what) + ": null cache");
+    if (int rc = check_device(c, what)) return rc;
+    if (int rc = check_seq(c, seq)) return rc;
+    if (layer < 0 || layer >= c->cfg.num_layers) return fail(KVC_ERR_INVALID, std::string(what) + ": bad layer");
+    if (first < 0 || n < 0 || (int64_t)first + n > c->lens[seq])
+        return fail(KVC_ERR_INVALID, std::string(what) + ": positions outside the reserved length");
+    if (n == 0) return KVC_OK;
+    if (!k || !v || !aligned16(k) || !aligned16(v))
+        return fail(KVC_ERR_INVALID, std::string(what) + ": k / v must be non-null and 16-byte aligned");
+    TokenCopyArgs a;
+    a.pool_k = c->k_pool(layer);
+    a.pool_v = c->v_pool(layer);
+    a.pt_row = c->page_table() + (int64_t)seq * c->cfg.max_pages_per_seq;
+    a.num_pages = c->cfg.num_pages;
+    a.H_kv = c->cfg.num_kv_heads;
+    a.D = c->cfg.head_dim;
+    a.first_pos = first;
+    a.n = n;
+    a.tok_k = static_cast<uint16_t*>(k);
+    a.tok_v = static_cast<uint16_t*>(v);
+    a.to_pool = to_pool;
+    a.err = c->err;
+    KVD_CUDA(launch_token_copy(a, static_cast<cudaStream_t>(stream)));
+    return KVC_OK;
+}
+
+int kv_write_tokens(kv_cache* c, int32_t layer, int32_t seq, int32_t first_pos, int32_t n, const void* k,
+                    const void* v, void* stream)
+{
+    return token_copy(c, "kv_write_tokens", layer, seq, first_pos, n, const_cast<void*>(k), const_cast<void*>(v), 1,
+                      stream);
+}
+
+int kv_read_tokens(kv_cache* c, int32_t layer, int32_t seq, int32_t first_pos, int32_t n, void* k_out, void* v_out,
+                   void* stream)
+{
+    return token_copy(c, "kv_read_tokens", layer, seq, first_pos, n, k_out, v_out, 0, stream);
+}
+
+int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stream)
+{
+    if (!c || !seq_ids) return fail(KVC_ERR_INVALID, "kv_begin_step: null argument");
+    if (batch < 1 || batch > c->cfg.max_seqs) return fail(KVC_ERR_INVALID, "kv_begin_step: batch outside 1 .. max_seqs");
+    if (++c->stamp_gen == 0) {
+        std::fill(c->stamp.begin(), c->stamp.end(), 0u);
+        c->stamp_gen = 1;
+    }
+    int64_t need = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t s = seq_ids[b];
+        if (int rc = check_seq(c, s)) return rc;
+        if (c->stamp[s] == c->stamp_gen) return fail(KVC_ERR_INVALID, "kv_begin_step: sequence listed twice");
+        c->stamp[s] = c->stamp_gen;
+        const int64_t len = c->lens[s];
+        if ((len + 1 + kPageSize - 1) / kPageSize > c->cfg.max_pages_per_seq)
+            return fail(KVC_ERR_INVALID, "kv_begin_step: page-table row too short");
+        if (len % kPageSize == 0) ++need;
+    }
+    if (need > (int64_t)c->free_stack.size()) return fail(KVC_ERR_OOM, "kv_begin_step: page pool exhausted");
+
+    // Size the plan from the lengths after this step, before changing anything.
+    int64_t total_units = 0;
+    for (int32_t b = 0; b < batch; ++b)
+        total_units += (int64_t)((c->lens[seq_ids[b]] + 1 + kPageSize - 1) / kPageSize) * c->cfg.num_kv_heads;
+    const int32_t C = c->split_override ? c->split_override : auto_split_pages(c, total_units);
+    int64_t entries = 0, total_full = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int64_t np = (c->lens[seq_ids[b]] + 1 + kPageSize - 1) / kPageSize;
+        total_full += np / C;
+        entries += np / C + (np % C ? 1 : 0);
+    }
+    if (!c->host_only)
+        if (int rc = grow_scratch(c, entries, entries * c->cfg.num_kv_heads, static_cast<cudaStream_t>(stream)))
+            return rc;
+
+    // Host mirror: every sequence of the batch gets position len.
+    std::vector<int32_t> new_page((size_t)batch, -1);
+    for (int32_t b = 0; b < batch; ++b) {
+        const int32_t s = seq_ids[b];
+        if (c->lens[s] % kPageSize == 0) {
+            new_page[b] = c->pop_page();
+            c->pages[s].push_back(new_page[b]);
+        }
+        c->lens[s] += 1;
+    }
+    c->step_active = false;
+    if (!c->host_only) {
+        cudaStream_t st = static_cast<cudaStream_t>(stream);
+        StepPatch patch;
+        PlanArgs pa;
+        pa.batch = batch;
+        pa.chunk_pages = C;
+        pa.max_pages = c->cfg.max_pages_per_seq;
+        pa.step_seq = c->step_seq;
+        pa.seq_len = c->seq_len_dev();
+        pa.page_table = c->page_table();
+        pa.plan = c->plan;
+        pa.err = c->err;
+        for (int32_t b0 = 0; b0 < batch; b0 += kPatchMax) {
+            const int32_t n = std::min(kPatchMax, batch - b0);
+            patch.n = n;
+            patch.b0 = b0;
+            for (int32_t i = 0; i < n; ++i) {
+                patch.seq[i] = seq_ids[b0 + i];
+                patch.new_len[i] = c->lens[seq_ids[b0 + i]];
+                patch.new_page[i] = new_page[b0 + i];
+            }
+            pa.build = (b0 + n == batch) ? 1 : 0;
+            KVD_CUDA(launch_step(patch, pa, (int32_t)total_full, st));
+        }
+    }
+    c->step_active = true;
+    c->step_batch = batch;
+    c->step_entries = (int32_t)entries;
+    return KVC_OK;
+}
+
+static int check_step(kv_cache* c, const char* what, int32_t layer, int32_t batch)
+{
+    if (!c) return fail(KVC_ERR_INVALID, std::string(what) + ": null cache");
+    if (int rc = check_device(c, what)) return rc;
+    if (!c->step_active) return fail(KVC_ERR_INVALID, std::string(what) + ": no decode step is active");
+    if (batch != c->step_batch) return fail(KVC_ERR_INVALID, std::string(what) + ": batch differs from the step's");
+    if (layer < 0 || layer >= c->cfg.num_layers) return fail(KVC_ERR_INVALID, std::string(what) + ": bad layer");
+    return KVC_OK;
+}
+
+int kv_append(kv_cache* c, int32_t layer, int32_t batch, const void* k_new, const void* v_new, void* stream)
+{
+    if (int rc = check_step(c, "kv_append", layer, batch)) return rc;
+    if (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new))
+        return fail(KVC_ERR_INVALID, "kv_append: k_new / v_new must be non-null and 16-byte aligned");
+    AppendArgs a;
+    a.pool_k = c->k_pool(layer);
+    a.pool_v = c->v_pool(layer);
+    a.k_new = static_cast<const uint16_t*>(k_new);
+    a.v_new = static_cast<const uint16_t*>(v_new);
+    a.step_seq = c->step_seq;
+    a.seq_len = c->seq_len_dev();
+    a.page_table = c->page_table();
+    a.num_pages = c->cfg.num_pages;
+    a.batch = batch;
+    a.H_kv = c->cfg.num_kv_heads;
+    a.D = c->cfg.head_dim;
+    a.max_pages = c->cfg.max_pages_per_seq;
+    a.err = c->err;
+    KVD_CUDA(launch_append(a, static_cast<cudaStream_t>(stream)));
+    return KVC_OK;
+}
+
+int decode_attention(kv_cache* c, int32_t layer, int32_t batch, const void* q, void* out, float softmax_scale,
+                     void* stream)
+{
+    if (int rc = check_step(c, "decode_attention", layer, batch)) return rc;
+    if (!q || !out || !aligned16(q) || !aligned16(out))
+        return fail(KVC_ERR_INVALID, "decode_attention: q / out must be non-null and 16-byte aligned");
+    if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale))
+        return fail(KVC_ERR_INVALID, "decode_attention: softmax_scale must be finite");
+    const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)c->cfg.head_dim);
+    DecodeParams p;
+    p.q = static_cast<const uint16_t*>(q);
+    p.out = static_cast<uint16_t*>(out);
+    p.page_table = c->page_table();
+    p.plan = c->plan;
+    p.part_o = c->part_o;
+    p.part_ml = c->part_ml;
+    p.tickets = c->tickets;
+    p.queue = c->queue;
+    p.err = c->err;
+    p.num_pages = c->cfg.num_pages;
+    p.n_items = c->step_entries * c->cfg.num_kv_heads;
+    p.H_kv = c->cfg.num_kv_heads;
+    p.H_q = c->cfg.num_q_heads;
+    p.G = c->group;
+    p.max_pages = c->cfg.max_pages_per_seq;
+    p.scale_log2 = scale * 1.4426950408889634f;
+    const int64_t resident = (int64_t)c->num_sms * std::max(1, c->variant.ctas_per_sm);
+    const int64_t want = (p.n_items + c->variant.warps - 1) / c->variant.warps;
+    const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
+    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, grid, c->tmaps[2 * layer], c->tmaps[2 * layer + 1], p,
+                           static_cast<cudaStream_t>(stream)));
+    return KVC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,118 @@
+// Internal declarations shared by the host library (kvd_host.cpp) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvd {
+
+constexpr int kPageSize = 16;          // tokens per page (the only supported P)
+constexpr int kMaxGroup = 8;           // query heads per KV head handled by one MMA N-tile
+constexpr int kMaxSplitPages = 64;     // pages per work item (two page-id registers per lane)
+constexpr int kPatchMax = 1024;        // step entries carried in one launch's parameters
+constexpr int kScatterMax = 2048;      // int32 updates carried in one launch's parameters
+
+// One work item of a step's split plan: consecutive pages [first_page,
+// first_page + n_pages) of batch row b.  Items are expanded over the H_kv
+// heads at launch time: item = entry * H_kv + g.
+struct PlanEntry {
+    int32_t b;          // batch row (q / out row)
+    int32_t seq;        // sequence id (page-table row)
+    int32_t len;        // tokens attended, including this step's token
+    int32_t first_page; // first logical page of the item
+    int32_t n_pages;    // pages of the item, 1 .. kMaxSplitPages
+    int32_t chunk;      // index of the item among the row's items
+    int32_t n_chunks;   // items of the row
+    int32_t slot_base;  // first partial slot of the row; slot = (slot_base + chunk) * H_kv + g
+};
+
+// Per-step update, passed by value in kernel parameters.
+struct StepPatch {
+    int32_t n;                     // entries in this launch
+    int32_t b0;                    // batch row of entry 0
+    int32_t seq[kPatchMax];
+    int32_t new_len[kPatchMax];
+    int32_t new_page[kPatchMax];   // page taken for position new_len-1, or -1
+};
+
+struct PlanArgs {
+    int32_t build;       // build the plan in this launch (last launch of a step)
+    int32_t batch;
+    int32_t chunk_pages; // C
+    int32_t max_pages;   // page-table row length
+    int32_t* step_seq;   // [max_seqs] batch row -> sequence id
+    int32_t* seq_len;    // [max_seqs]
+    int32_t* page_table; // [max_seqs][max_pages]
+    PlanEntry* plan;     // [n_entries]
+    int32_t* err;
+};
+
+struct ScatterI32 {
+    int32_t n;
+    int32_t idx[kScatterMax];
+    int32_t val[kScatterMax];
+};
+
+struct TokenCopyArgs {
+    uint16_t* pool_k;         // layer pool base [num_pages][H_kv][P][D]
+    uint16_t* pool_v;
+    const int32_t* pt_row;    // page-table row of the sequence (device)
+    int64_t num_pages;
+    int32_t H_kv, D;
+    int32_t first_pos, n;
+    uint16_t* tok_k;          // [n][H_kv][D] logical order
+    uint16_t* tok_v;
+    int32_t to_pool;          // 1: tokens -> pool, 0: pool -> tokens
+    int32_t* err;
+};
+
+struct AppendArgs {
+    uint16_t* pool_k;
+    uint16_t* pool_v;
+    const uint16_t* k_new;    // [B][H_kv][D]
+    const uint16_t* v_new;
+    const int32_t* step_seq;
+    const int32_t* seq_len;
+    const int32_t* page_table;
+    int64_t num_pages;
+    int32_t batch, H_kv, D, max_pages;
+    int32_t* err;
+};
+
+struct DecodeParams {
+    const uint16_t* q;        // [B][H_q][D] bf16
+    uint16_t* out;            // [B][H_q][D] bf16
+    const int32_t* page_table;
+    const PlanEntry* plan;
+    float* part_o;            // [slots][G][D]
+    float2* part_ml;          // [slots][G]  (running max in log2 units, sum)
+    int32_t* tickets;         // [batch][H_kv]
+    uint32_t* queue;          // [0] next item, [1] warps finished
+    int32_t* err;
+    int64_t num_pages;
+    int32_t n_items;
+    int32_t H_kv, H_q, G, max_pages;
+    float scale_log2;         // softmax scale * log2(e)
+};
+
+// ---- launchers (return cudaGetLastError() of the launch) -----------------
+cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st);
+// total_full: number of full-size items of the plan (the host knows it).
+cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, int32_t total_full,
+                        cudaStream_t st);
+cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
+
+// Decode attention: variant chosen by (D, G == 1).
+struct DecodeVariant {
+    int warps;        // warps per CTA
+    int smem_bytes;   // dynamic shared memory per CTA
+    int ctas_per_sm;  // occupancy at that shared memory
+};
+cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v);
+cudaError_t launch_decode(int D, bool gqa, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+                          const DecodeParams& p, cudaStream_t st);
+
+}  // namespace kvd

@@ -1,0 +1,210 @@
+"""ctypes binding of libkvdecode.so (declared in include/kvdecode.h).
+
+Argument marshalling only: every step of the decode path runs in the CUDA
+library.  Functions keep the C names; pointer arguments accept torch tensors
+(their ``data_ptr()``), plain integers or None, and ``stream`` accepts a
+``torch.cuda.Stream``, a raw handle or None (the legacy default stream).
+If the library has not been built, loading fails loudly: there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libkvdecode.so")
+
+KVC_OK = 0
+KVC_ERR_INVALID = -1
+KVC_ERR_OOM = -2
+KVC_ERR_CUDA = -3
+KVC_ERR_PAGE_TABLE = -4
+KVC_ERR_UNSUPPORTED = -5
+KVC_ERR_DEVICE = -6
+KVC_FLAG_HOST_ONLY = 1
+KVC_DEVERR_PAGE_RANGE = 1
+KVC_DEVERR_WAIT_TIMEOUT = 2
+KVC_DEVERR_SEQ_RANGE = 4
+
+_NAMES = {KVC_ERR_INVALID: "INVALID", KVC_ERR_OOM: "OOM", KVC_ERR_CUDA: "CUDA",
+          KVC_ERR_PAGE_TABLE: "PAGE_TABLE", KVC_ERR_UNSUPPORTED: "UNSUPPORTED",
+          KVC_ERR_DEVICE: "DEVICE"}
+
+
+class KVDecodeError(RuntimeError):
+    def __init__(self, code: int, fn: str, msg: str):
+        super().__init__(f"{fn} -> KVC_ERR_{_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+class kvc_config(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int32), ("num_q_heads", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("max_seqs", ctypes.c_int32),
+                ("max_pages_per_seq", ctypes.c_int32), ("flags", ctypes.c_int32),
+                ("num_pages", ctypes.c_int64)]
+
+
+class kvc_stats(ctypes.Structure):
+    _fields_ = [("kv_bytes_allocated", ctypes.c_int64), ("pool_bytes", ctypes.c_int64),
+                ("pages_in_use", ctypes.c_int64), ("free_pages", ctypes.c_int64),
+                ("live_seqs", ctypes.c_int32), ("device_error", ctypes.c_int32)]
+
+
+_lib = None
+_P = ctypes.c_void_p
+_I32 = ctypes.c_int32
+_I64 = ctypes.c_int64
+_SIGS = {
+    "kv_cache_create": [ctypes.POINTER(kvc_config), _P, ctypes.POINTER(_P)],
+    "kv_cache_destroy": [_P],
+    "kv_cache_set_page_order": [_P, _P, _I64],
+    "kv_cache_query": [_P, ctypes.POINTER(kvc_stats)],
+    "kv_cache_pool": [_P, _I32, ctypes.POINTER(_P), ctypes.POINTER(_P)],
+    "kv_cache_set_split_pages": [_P, _I32],
+    "kv_seq_create": [_P, ctypes.POINTER(_I32)],
+    "kv_seq_reserve": [_P, _I32, _I32, _P],
+    "kv_seq_free": [_P, _I32, _P],
+    "kv_seq_info": [_P, _I32, ctypes.POINTER(_I32), _P, _I32, ctypes.POINTER(_I32)],
+    "kv_write_tokens": [_P, _I32, _I32, _I32, _I32, _P, _P, _P],
+    "kv_read_tokens": [_P, _I32, _I32, _I32, _I32, _P, _P, _P],
+    "kv_begin_step": [_P, _I32, _P, _P],
+    "kv_append": [_P, _I32, _I32, _P, _P, _P],
+    "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
+}
+
+
+def load():
+    """Load libkvdecode.so (raises if it is missing)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run `python -c \"import __graft_entry__ as g; "
+                               f"g.build()\"` (needs nvcc)")
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, args in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_int
+        lib.kv_last_error.argtypes = []
+        lib.kv_last_error.restype = ctypes.c_char_p
+        _lib = lib
+    return _lib
+
+
+def _ptr(x):
+    if x is None:
+        return None
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    if isinstance(x, ctypes.Array):
+        return ctypes.addressof(x)
+    return int(x)
+
+
+def _stream(s):
+    if s is None:
+        return None
+    if hasattr(s, "cuda_stream"):
+        return s.cuda_stream
+    return int(s)
+
+
+def _check(rc: int, fn: str):
+    if rc != KVC_OK:
+        raise KVDecodeError(rc, fn, load().kv_last_error().decode())
+
+
+def _i32_array(values):
+    vals = [int(v) for v in values]
+    return (ctypes.c_int32 * len(vals))(*vals)
+
+
+# ---------------------------------------------------------------- C names
+def kv_cache_create(cfg: kvc_config, stream=None):
+    h = _P()
+    _check(load().kv_cache_create(ctypes.byref(cfg), _stream(stream), ctypes.byref(h)), "kv_cache_create")
+    return h
+
+
+def kv_cache_destroy(h):
+    _check(load().kv_cache_destroy(h), "kv_cache_destroy")
+
+
+def kv_cache_set_page_order(h, order):
+    arr = _i32_array(order)
+    _check(load().kv_cache_set_page_order(h, ctypes.addressof(arr), len(arr)), "kv_cache_set_page_order")
+
+
+def kv_cache_query(h, raise_on_device_error: bool = True) -> kvc_stats:
+    s = kvc_stats()
+    rc = load().kv_cache_query(h, ctypes.byref(s))
+    if rc != KVC_OK and (raise_on_device_error or rc not in (KVC_ERR_PAGE_TABLE, KVC_ERR_DEVICE)):
+        _check(rc, "kv_cache_query")
+    return s
+
+
+def kv_cache_pool(h, layer: int):
+    k, v = _P(), _P()
+    _check(load().kv_cache_pool(h, layer, ctypes.byref(k), ctypes.byref(v)), "kv_cache_pool")
+    return k.value, v.value
+
+
+def kv_cache_set_split_pages(h, pages: int):
+    _check(load().kv_cache_set_split_pages(h, pages), "kv_cache_set_split_pages")
+
+
+def kv_seq_create(h) -> int:
+    s = _I32()
+    _check(load().kv_seq_create(h, ctypes.byref(s)), "kv_seq_create")
+    return s.value
+
+
+def kv_seq_reserve(h, seq: int, n_tokens: int, stream=None):
+    _check(load().kv_seq_reserve(h, seq, n_tokens, _stream(stream)), "kv_seq_reserve")
+
+
+def kv_seq_free(h, seq: int, stream=None):
+    _check(load().kv_seq_free(h, seq, _stream(stream)), "kv_seq_free")
+
+
+def kv_seq_info(h, seq: int):
+    """Returns (length, [page ids in logical order])."""
+    ln, npg = _I32(), _I32()
+    _check(load().kv_seq_info(h, seq, ctypes.byref(ln), None, 0, ctypes.byref(npg)), "kv_seq_info")
+    buf = (ctypes.c_int32 * max(1, npg.value))()
+    _check(load().kv_seq_info(h, seq, ctypes.byref(ln), ctypes.addressof(buf), npg.value, ctypes.byref(npg)),
+           "kv_seq_info")
+    return ln.value, list(buf[:npg.value])
+
+
+def kv_write_tokens(h, layer: int, seq: int, first_pos: int, n: int, k, v, stream=None):
+    _check(load().kv_write_tokens(h, layer, seq, first_pos, n, _ptr(k), _ptr(v), _stream(stream)),
+           "kv_write_tokens")
+
+
+def kv_read_tokens(h, layer: int, seq: int, first_pos: int, n: int, k_out, v_out, stream=None):
+    _check(load().kv_read_tokens(h, layer, seq, first_pos, n, _ptr(k_out), _ptr(v_out), _stream(stream)),
+           "kv_read_tokens")
+
+
+def kv_begin_step(h, seq_ids, stream=None):
+    arr = _i32_array(seq_ids)
+    _check(load().kv_begin_step(h, len(arr), ctypes.addressof(arr), _stream(stream)), "kv_begin_step")
+
+
+def kv_append(h, layer: int, batch: int, k_new, v_new, stream=None):
+    _check(load().kv_append(h, layer, batch, _ptr(k_new), _ptr(v_new), _stream(stream)), "kv_append")
+
+
+def decode_attention(h, layer: int, batch: int, q, out, softmax_scale: float = 0.0, stream=None):
+    _check(load().decode_attention(h, layer, batch, _ptr(q), _ptr(out), float(softmax_scale), _stream(stream)),
+           "decode_attention")
+
+
+def make_config(num_layers, num_q_heads, num_kv_heads, head_dim, num_pages, max_seqs, max_pages_per_seq,
+                page_size=16, flags=0) -> kvc_config:
+    return kvc_config(num_layers=num_layers, num_q_heads=num_q_heads, num_kv_heads=num_kv_heads,
+                      head_dim=head_dim, page_size=page_size, max_seqs=max_seqs,
+                      max_pages_per_seq=max_pages_per_seq, flags=flags, num_pages=num_pages)

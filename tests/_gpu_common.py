@@ -1,0 +1,115 @@
+"""Shared pieces of the GPU parity tests: a decode session that also keeps the
+host copy of everything the cache should hold, so the oracle can be fed the
+same logical-order K/V."""
+import numpy as np
+import torch
+
+import oracle
+from paper_2603_12707_gb300 import kvdecode as kd
+from paper_2603_12707_gb300 import workloads as wl
+from paper_2603_12707_gb300.harness import DecodeSession
+
+
+def u16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+class _CAI:
+    """Expose a raw device allocation to torch (int16 view) for read-back."""
+
+    def __init__(self, ptr, shape):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": "<i2", "data": (int(ptr), False),
+                                         "version": 3, "strides": None}
+
+
+def device_pool(sess: DecodeSession, layer: int):
+    """Raw K and V pools of one layer as uint16 [num_pages, H_kv, P, d] host arrays."""
+    kp, vp = kd.kv_cache_pool(sess.h, layer)
+    c = sess.cfg
+    shape = (sess.num_pages, c.num_kv_heads, c.page_size, c.head_dim)
+    k = torch.as_tensor(_CAI(kp, shape), device="cuda")
+    v = torch.as_tensor(_CAI(vp, shape), device="cuda")
+    torch.cuda.synchronize()
+    return u16(k), u16(v)
+
+
+class Tracked:
+    """A DecodeSession plus host copies of each layer pool's logical content."""
+
+    def __init__(self, cfg, extra_tokens=8, lens=None, split_pages=0, layers_filled=None, keep_host=True,
+                 keep_rows=None):
+        self.cfg = cfg
+        self.sess = DecodeSession(cfg, extra_tokens=extra_tokens, lens=lens, split_pages=split_pages)
+        self.keep_host = keep_host
+        self.keep_rows = list(range(cfg.batch)) if keep_rows is None else list(keep_rows)
+        self.layers_filled = list(range(cfg.phys_layers)) if layers_filled is None else list(layers_filled)
+        self.sess.fill_prefix(self.layers_filled)
+        # host logical content per (phys layer, batch row): list of token rows [H_kv, d]
+        self.k = {}
+        self.v = {}
+        if keep_host:
+            for l in self.layers_filled:
+                for b in self.keep_rows:
+                    n = int(self.sess.lens0[b])
+                    self.k[(l, b)] = list(u16(wl.kv_block(cfg, l, b, n, "k", "cuda"))) if n else []
+                    self.v[(l, b)] = list(u16(wl.kv_block(cfg, l, b, n, "v", "cuda"))) if n else []
+        self.step = -1
+
+    def begin_step(self):
+        self.sess.begin_step()
+        self.step += 1
+
+    def run_layer(self, layer, scale=0.0):
+        """Append + attend one logical layer; returns (out bf16 tensor, q, k_new, v_new)."""
+        cfg = self.cfg
+        q, kn, vn = wl.step_inputs(cfg, self.step, layer, "cuda")
+        out = torch.empty_like(q)
+        self.sess.append(layer, kn, vn)
+        self.sess.attend(layer, q, out, scale)
+        if self.keep_host:
+            p = self.sess.phys(layer)
+            kh, vh = u16(kn), u16(vn)
+            for b in self.keep_rows:
+                pos = int(self.sess.lens[b]) - 1
+                for store, val in ((self.k, kh[b]), (self.v, vh[b])):
+                    rows = store[(p, b)]
+                    if pos == len(rows):
+                        rows.append(val)
+                    else:
+                        rows[pos] = val
+        return out, q, kn, vn
+
+    def oracle(self, layer, q, rows=None, scale=None):
+        """float64 oracle output for the given batch rows of one layer."""
+        p = self.sess.phys(layer)
+        rows = list(range(self.cfg.batch)) if rows is None else list(rows)
+        lens = [len(self.k[(p, b)]) for b in rows]
+        k = np.concatenate([np.stack(self.k[(p, b)]) for b in rows])
+        v = np.concatenate([np.stack(self.v[(p, b)]) for b in rows])
+        qh = u16(q)[rows]
+        ref = oracle.decode_attention(qh, lens, k, v, scale=scale)
+        vmax = np.array([np.abs(oracle.bf16_to_f64(np.stack(self.v[(p, b)]))).max() for b in rows])
+        return ref, vmax
+
+    def close(self):
+        st = self.sess.query()
+        assert st.device_error == 0
+        self.sess.close()
+
+
+def bf16_to_f64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().double().numpy()
+
+
+def assert_close(got, ref, vmax, gqa: bool, what=""):
+    """Spec bound (max |err| <= 2e-2, mean |err| <= 2e-3) and the bound
+    derived from the arithmetic: bf16 rounding of the output (2^-8 relative),
+    bf16 rounding of the softmax weights fed to the P.V MMA (2^-9 * max|v|,
+    GQA only) and fp32 accumulation (1e-5 * max|v|)."""
+    err = np.abs(got - ref)
+    assert err.max() <= 2e-2, (what, err.max())
+    assert err.mean() <= 2e-3, (what, err.mean())
+    w = (2.0 ** -9 if gqa else 0.0) + 1e-5
+    bound = 2.0 ** -8 * np.abs(ref) + w * vmax[:, None, None]
+    bad = err > bound
+    assert not bad.any(), (what, int(bad.sum()), float((err - bound).max()), np.argwhere(bad)[:5].tolist())

@@ -1,0 +1,207 @@
+"""GPU parity of the CUDA path against the float64 oracle, through the C ABI.
+
+* kv_append and the prefix write: bit-exact pool contents and page tables.
+* decode_attention: every output element against the oracle, on small
+  configs that span several pages, splits and a ragged tail, on the edge
+  cases (a fresh sequence attending one token, page-boundary lengths, one
+  page per split, unsplit rows), and on sampled rows of the five workload
+  shapes at full size in the launch configuration the bench uses.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import PagePoolModel
+from paper_2603_12707_gb300 import kvdecode as kd
+from paper_2603_12707_gb300 import workloads as wl
+
+from _gpu_common import Tracked, assert_close, bf16_to_f64, device_pool, u16
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True, scope="module")
+def _lib(kvlib):
+    assert torch.cuda.is_available()
+    yield
+
+
+def _model_for(sess):
+    c = sess.cfg
+    m = PagePoolModel(sess.num_pages, c.page_size, c.batch, sess.max_pages)
+    order = wl.page_order(c, sess.num_pages)
+    if order is not None:
+        m.set_page_order(order)
+    for _ in range(c.batch):
+        m.seq_create()
+    for i, n in wl.reserve_schedule(c, sess.lens0):
+        m.seq_reserve(i, n)
+    return m
+
+
+# ---------------------------------------------------------------- kv_append
+@pytest.mark.parametrize("cfg", [
+    wl.CONFIGS["tiny"],
+    wl.custom("gqa128", 2, 14, 2, 128, 5, lens=[0, 15, 16, 17, 40], page_order="interleaved"),
+    wl.custom("mha64", 1, 4, 4, 64, 3, lens=[31, 32, 1], page_order="shuffled", seed=9),
+])
+def test_prefix_write_and_append_are_bit_exact(cfg):
+    t = Tracked(cfg, extra_tokens=40)
+    sess = t.sess
+    model = _model_for(sess)
+    for step in range(3):
+        t.begin_step()
+        model.begin_step(list(range(cfg.batch)))
+        for layer in range(cfg.num_layers):
+            t.run_layer(layer)
+    torch.cuda.synchronize()
+    # page tables: library == oracle allocator model, entry for entry
+    for b, seq in enumerate(sess.seq_ids):
+        ln, pages = kd.kv_seq_info(sess.h, seq)
+        assert ln == model.lens[b] and pages == model.pages[b]
+    # pools: the oracle scatters the same logical rows through the model's tables
+    for l in range(cfg.phys_layers):
+        shape = (sess.num_pages, cfg.num_kv_heads, cfg.page_size, cfg.head_dim)
+        ek, ev = np.zeros(shape, np.uint16), np.zeros(shape, np.uint16)
+        for b in range(cfg.batch):
+            row = np.array(model.pages[b], np.int32)
+            if len(t.k[(l, b)]):
+                oracle.kv_scatter(ek, row, 0, np.stack(t.k[(l, b)]), cfg.page_size)
+                oracle.kv_scatter(ev, row, 0, np.stack(t.v[(l, b)]), cfg.page_size)
+        gk, gv = device_pool(sess, l)
+        assert np.array_equal(gk, ek) and np.array_equal(gv, ev)
+        # read-back through the ABI returns the logical rows
+        for b, seq in enumerate(sess.seq_ids):
+            n = int(sess.lens[b])
+            ko = torch.empty((n, cfg.num_kv_heads, cfg.head_dim), dtype=torch.bfloat16, device="cuda")
+            vo = torch.empty_like(ko)
+            kd.kv_read_tokens(sess.h, l, seq, 0, n, ko, vo)
+            assert np.array_equal(u16(ko), np.stack(t.k[(l, b)]))
+            assert np.array_equal(u16(vo), np.stack(t.v[(l, b)]))
+    t.close()
+
+
+# ---------------------------------------------------------- decode: small
+SMALL = [
+    # name, Hq, Hkv, d, lens (cached before the first step)
+    ("mha64", 8, 8, 64, [0, 1, 15, 16, 17, 95, 130]),
+    ("mha128", 4, 4, 128, [0, 15, 16, 31, 200, 513]),
+    ("gqa7_128", 28, 4, 128, [0, 1, 16, 47, 300]),
+    ("gqa7_64", 14, 2, 64, [3, 16, 33, 250]),
+    ("gqa8_64", 8, 1, 64, [5, 64, 129]),
+    ("gqa2_128", 4, 2, 128, [17, 100, 1000]),
+]
+
+
+@pytest.mark.parametrize("split", [0, 1, 3, 64])
+@pytest.mark.parametrize("name,Hq,Hkv,d,lens", SMALL)
+def test_decode_matches_oracle_small(name, Hq, Hkv, d, lens, split):
+    cfg = wl.custom(name, 2, Hq, Hkv, d, len(lens), lens=lens, seed=31 + Hq + d, page_order="shuffled")
+    t = Tracked(cfg, extra_tokens=20, split_pages=split)
+    for step in range(3):
+        t.begin_step()
+        for layer in range(cfg.num_layers):
+            out, q, _, _ = t.run_layer(layer)
+            torch.cuda.synchronize()
+            ref, vmax = t.oracle(layer, q)
+            assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv, what=(name, split, step, layer))
+    t.close()
+
+
+def test_custom_softmax_scale():
+    cfg = wl.custom("scale", 1, 14, 2, 128, 3, lens=[10, 40, 90], seed=5)
+    t = Tracked(cfg)
+    t.begin_step()
+    out, q, _, _ = t.run_layer(0, scale=0.37)
+    torch.cuda.synchronize()
+    ref, vmax = t.oracle(0, q, scale=0.37)
+    assert_close(bf16_to_f64(out), ref, vmax, gqa=True)
+    t.close()
+
+
+def test_single_token_context_returns_appended_v():
+    """A sequence with nothing cached attends only its new token: out == v_new
+    exactly (weights are exactly 1, and bf16 -> fp32 -> bf16 is lossless)."""
+    for Hq, Hkv, d in ((8, 8, 64), (28, 4, 128)):
+        cfg = wl.custom("one", 1, Hq, Hkv, d, 3, lens=[0, 0, 0], seed=3)
+        t = Tracked(cfg)
+        t.begin_step()
+        out, q, kn, vn = t.run_layer(0)
+        torch.cuda.synchronize()
+        G = Hq // Hkv
+        expect = vn.repeat_interleave(G, dim=1)
+        assert torch.equal(out, expect)
+        t.close()
+
+
+def test_page_order_does_not_change_results():
+    """Same logical content in different physical pages: bit-identical output."""
+    outs = []
+    for order in ("sequential", "shuffled", "interleaved"):
+        cfg = wl.custom("perm", 1, 28, 4, 128, 4, lens=[100, 37, 260, 16], seed=77, page_order=order)
+        t = Tracked(cfg, keep_host=False)
+        t.begin_step()
+        out, _, _, _ = t.run_layer(0)
+        torch.cuda.synchronize()
+        outs.append(out.clone())
+        t.close()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+def test_split_size_changes_only_rounding():
+    res = {}
+    for split in (1, 4, 64):
+        cfg = wl.custom("split", 1, 8, 8, 128, 3, lens=[700, 33, 1023], seed=13)
+        t = Tracked(cfg, split_pages=split, keep_host=False)
+        t.begin_step()
+        out, _, _, _ = t.run_layer(0)
+        torch.cuda.synchronize()
+        res[split] = bf16_to_f64(out)
+        t.close()
+    for s in (1, 4):
+        d = np.abs(res[s] - res[64])
+        assert d.max() <= 2.0 ** -7 * np.abs(res[64]).max()
+
+
+def test_step_and_attention_errors_do_not_launch():
+    cfg = wl.custom("err", 1, 8, 8, 64, 2, lens=[5, 9], seed=1)
+    t = Tracked(cfg, keep_host=False)
+    q = torch.zeros((2, 8, 64), dtype=torch.bfloat16, device="cuda")
+    out = torch.empty_like(q)
+    with pytest.raises(kd.KVDecodeError):           # no step yet
+        kd.decode_attention(t.sess.h, 0, 2, q, out)
+    t.begin_step()
+    with pytest.raises(kd.KVDecodeError):           # wrong batch
+        kd.decode_attention(t.sess.h, 0, 1, q, out)
+    with pytest.raises(kd.KVDecodeError):           # bad layer
+        kd.kv_append(t.sess.h, 3, 2, q, q)
+    with pytest.raises(kd.KVDecodeError):           # misaligned pointer
+        kd.decode_attention(t.sess.h, 0, 2, q.data_ptr() + 2, out)
+    t.close()
+
+
+# ------------------------------------------------------- decode: full size
+FULL = [
+    # config, logical layers checked, sampled batch rows
+    ("tiny", [0], None),
+    ("llava", [0, 17, 31], [0, 1, 2, 63]),
+    ("qwen", [0, 27], [0, 5, 31]),
+    ("long", [0, 27], [0, 7]),
+    ("ragged", [0, 9, 31], [0, 100, 255]),
+]
+
+
+@pytest.mark.parametrize("name,layers,rows", FULL)
+def test_decode_matches_oracle_full_size(name, layers, rows):
+    cfg = wl.CONFIGS[name]
+    phys = sorted({l % cfg.phys_layers for l in layers})
+    t = Tracked(cfg, extra_tokens=4, layers_filled=phys, keep_rows=rows)
+    t.begin_step()
+    for layer in layers:
+        out, q, _, _ = t.run_layer(layer)
+        torch.cuda.synchronize()
+        r = list(range(cfg.batch)) if rows is None else rows
+        ref, vmax = t.oracle(layer, q, rows=r)
+        assert_close(bf16_to_f64(out)[r], ref, vmax, gqa=cfg.group > 1, what=(name, layer))
+    t.close()
