@@ -190,6 +190,39 @@ KVC_API int kv_append(kv_cache *cache, int32_t layer, int32_t batch, const void 
 KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, const void *q, void *out,
                      float softmax_scale, void *stream);
 
+/* ------------------------------------------------ allocation-free decode -- */
+
+/* decode_attention for callers that may not allocate device memory while they
+ * serve: an engine plugin held to a memory budget fixed when the engine was
+ * built, a runtime whose device memory all belongs to another framework's
+ * allocator, a decode thread that must not take the allocator's locks.  Such a
+ * caller owns the K/V pools and the page table and passes them in; this call
+ * allocates nothing (no cudaMalloc, cudaMallocAsync, cudaFree or allocating
+ * library routine).  The paper has no counterpart: it is a convenience of this
+ * library, computing the same attention as decode_attention.
+ *   k_pool, v_pool  device, [num_pages][num_kv_heads][16][head_dim] bf16 (the
+ *                   layout kv_cache_pool exposes), 16-byte aligned
+ *   page_table      device, [batch][max_pages] int32: row b lists the pages of
+ *                   sequence b in logical order
+ *   lens            host, [batch]: tokens attended by row b, 1 .. max_pages*16
+ *   q, out          device, [batch][num_q_heads][head_dim] bf16
+ *   device_error    device int32 that receives KVC_DEVERR_* bits (OR-ed, never
+ *                   cleared by this call), or NULL to discard them
+ * Work space is a 16 MiB array in this library's device code, held by every
+ * GPU that loads the library until the process exits.  batch <= 1024;
+ * KVC_ERR_UNSUPPORTED if the batch's split plan and partial results need
+ * more than 16 MiB even at the largest split (64 pages).  The first call on
+ * each device looks up the array's device address (cudaGetSymbolAddress);
+ * make that first call before any stream capture.  Every call uses the same
+ * array and clears the counters it needs at its start, so calls that overlap
+ * on the GPU race: order them on one stream.  Same shape limits as
+ * kv_cache_create (head_dim 64 or 128, G <= 8, 16-token pages). */
+KVC_API int decode_attention_noalloc(const void *k_pool, const void *v_pool, int64_t num_pages,
+                                     int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                     int32_t batch, const int32_t *page_table, int32_t max_pages,
+                                     const int32_t *lens, const void *q, void *out,
+                                     float softmax_scale, int32_t *device_error, void *stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 KVC_API const char *kv_last_error(void);
 

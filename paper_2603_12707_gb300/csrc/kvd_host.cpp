@@ -52,6 +52,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 }  // namespace
 
+void kvd::set_last_error(const char* msg) { g_last_error = msg; }
+
 struct kv_cache {
     kvc_config cfg{};
     bool host_only = false;

@@ -97,6 +97,9 @@ struct DecodeParams {
     float scale_log2;         // softmax scale * log2(e)
 };
 
+// Message returned by kv_last_error() on the calling thread.
+void set_last_error(const char* msg);
+
 // ---- launchers (return cudaGetLastError() of the launch) -----------------
 cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st);
 // total_full: number of full-size items of the plan (the host knows it).

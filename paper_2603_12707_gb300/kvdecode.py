@@ -72,6 +72,8 @@ _SIGS = {
     "kv_begin_step": [_P, _I32, _P, _P],
     "kv_append": [_P, _I32, _I32, _P, _P, _P],
     "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
+    "decode_attention_noalloc": [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _I32, _P, _P, _P,
+                                 ctypes.c_float, _P, _P],
 }
 
 
@@ -201,6 +203,19 @@ def kv_append(h, layer: int, batch: int, k_new, v_new, stream=None):
 def decode_attention(h, layer: int, batch: int, q, out, softmax_scale: float = 0.0, stream=None):
     _check(load().decode_attention(h, layer, batch, _ptr(q), _ptr(out), float(softmax_scale), _stream(stream)),
            "decode_attention")
+
+
+def decode_attention_noalloc(k_pool, v_pool, num_pages: int, num_q_heads: int, num_kv_heads: int,
+                             head_dim: int, page_table, max_pages: int, lens, q, out,
+                             softmax_scale: float = 0.0, device_error=None, stream=None):
+    """Allocation-free decode attention over caller-owned pools and page
+    table; ``lens`` is a host sequence of attended token counts, one per row."""
+    arr = _i32_array(lens)
+    _check(load().decode_attention_noalloc(_ptr(k_pool), _ptr(v_pool), num_pages, num_q_heads, num_kv_heads,
+                                           head_dim, len(arr), _ptr(page_table), max_pages,
+                                           ctypes.addressof(arr), _ptr(q), _ptr(out), float(softmax_scale),
+                                           _ptr(device_error), _stream(stream)),
+           "decode_attention_noalloc")
 
 
 def make_config(num_layers, num_q_heads, num_kv_heads, head_dim, num_pages, max_seqs, max_pages_per_seq,
