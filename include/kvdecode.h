@@ -121,9 +121,11 @@ KVC_API int kv_cache_query(kv_cache *cache, kvc_stats *stats);
  * bf16), for inspection; owned by the cache. */
 KVC_API int kv_cache_pool(kv_cache *cache, int32_t layer, void **k_pool, void **v_pool);
 
-/* Override the split size (pages per work item of decode_attention) used
- * by later kv_begin_step calls; 0 restores the automatic choice.
- * Range 0 .. 64. */
+/* Override the target split size (pages per work item of decode_attention)
+ * used by later kv_begin_step calls; 0 restores the automatic choice.
+ * Range 0 .. 1024.  A row of n pages is cut into ceil(n / T') items of
+ * near-equal size, T' = max(T, ceil(n / 32)): never more than 32 items per
+ * (sequence, KV head). */
 KVC_API int kv_cache_set_split_pages(kv_cache *cache, int32_t pages);
 
 /* -------------------------------------------------------- sequences ------ */
@@ -209,9 +211,10 @@ KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, cons
  *   device_error    device int32 that receives KVC_DEVERR_* bits (OR-ed, never
  *                   cleared by this call), or NULL to discard them
  * Work space is a 16 MiB array in this library's device code, held by every
- * GPU that loads the library until the process exits.  batch <= 1024;
- * KVC_ERR_UNSUPPORTED if the batch's split plan and partial results need
- * more than 16 MiB even at the largest split (64 pages).  The first call on
+ * GPU that loads the library until the process exits.  batch <= 1024.
+ * Work items are enlarged until the split plan and partial results fit the
+ * 16 MiB (one item per row needs no partials at all);
+ * KVC_ERR_UNSUPPORTED if they still do not fit.  The first call on
  * each device looks up the array's device address (cudaGetSymbolAddress);
  * make that first call before any stream capture.  Every call uses the same
  * array and clears the counters it needs at its start, so calls that overlap

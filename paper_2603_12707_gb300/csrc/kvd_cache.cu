@@ -44,10 +44,11 @@ __device__ int block_exclusive_scan(int v, int* total)
 }
 
 // Apply the step's length / page-table updates; in the last launch of a step,
-// build the split plan: each batch row's pages cut into items of C pages,
-// full items first (in row order), then every row's shorter last item.
+// build the split plan: rows in the host's order (longest first when the
+// batch fits one launch), each row cut into row_chunks() items of near-equal
+// size, a row's items adjacent.
 __global__ void __launch_bounds__(1024)
-    step_kernel(const __grid_constant__ StepPatch patch, const PlanArgs a, int32_t total_full)
+    step_kernel(const __grid_constant__ StepPatch patch, const __grid_constant__ PlanArgs a)
 {
     for (int i = threadIdx.x; i < patch.n; i += blockDim.x) {
         const int seq = patch.seq[i], len = patch.new_len[i];
@@ -58,12 +59,12 @@ __global__ void __launch_bounds__(1024)
     }
     if (!a.build) return;
     __syncthreads();
-    const int C = a.chunk_pages;
-    int carry_full = 0, carry_rem = 0, carry_nch = 0;
+    int carry = 0;
     for (int base = 0; base < a.batch; base += blockDim.x) {
-        const int b = base + threadIdx.x;
-        int seq = 0, len = 0, np = 0;
-        if (b < a.batch) {
+        const int i = base + threadIdx.x;
+        int b = 0, seq = 0, len = 0, np = 0, nch = 0;
+        if (i < a.batch) {
+            b = a.use_order ? a.order[i] : i;
             seq = a.step_seq[b];
             len = a.seq_len[seq];
             if (len <= 0 || len > a.max_pages * kPageSize) {
@@ -71,26 +72,16 @@ __global__ void __launch_bounds__(1024)
                 len = 1;
             }
             np = (len + kPageSize - 1) / kPageSize;
+            nch = row_chunks(np, a.item_pages);
         }
-        const int full = np / C, rem = (np % C) ? 1 : 0, nch = full + rem;
-        int t_full, t_rem, t_nch;
-        const int ex_full = block_exclusive_scan(full, &t_full);
-        const int ex_rem = block_exclusive_scan(rem, &t_rem);
-        const int ex_nch = block_exclusive_scan(nch, &t_nch);
-        if (b < a.batch) {
-            const int slot_base = carry_nch + ex_nch;
-            for (int c = 0; c < full; ++c) {
-                PlanEntry e{b, seq, len, c * C, C, c, nch, slot_base};
-                a.plan[carry_full + ex_full + c] = e;
-            }
-            if (rem) {
-                PlanEntry e{b, seq, len, full * C, np - full * C, full, nch, slot_base};
-                a.plan[total_full + carry_rem + ex_rem] = e;
-            }
+        int total;
+        const int off = carry + block_exclusive_scan(nch, &total);
+        for (int c = 0; c < nch; ++c) {
+            int first, n;
+            chunk_range(np, nch, c, &first, &n);
+            a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
         }
-        carry_full += t_full;
-        carry_rem += t_rem;
-        carry_nch += t_nch;
+        carry += total;
     }
 }
 
@@ -163,10 +154,9 @@ cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t 
     return cudaGetLastError();
 }
 
-cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, int32_t total_full,
-                        cudaStream_t st)
+cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, cudaStream_t st)
 {
-    step_kernel<<<1, 1024, 0, st>>>(patch, plan, total_full);
+    step_kernel<<<1, 1024, 0, st>>>(patch, plan);
     return cudaGetLastError();
 }
 

@@ -3,9 +3,9 @@
 // Schedule.  A step's plan cuts every (sequence, KV head) into work items of
 // consecutive pages.  A persistent grid of warps pulls items from a global
 // counter; each warp runs its items independently:
-//   * one lane streams the item's (page, head) tiles of K and V into the
-//     warp's private ring of R shared-memory stages with 2-D TMA tile loads
-//     (128-byte swizzle, L2 evict-first), completing on one mbarrier per stage;
+//   * one lane streams (page, head) tiles of K and V into the warp's private
+//     ring of R shared-memory stages with 2-D TMA tile loads (128-byte
+//     swizzle, L2 evict-first), completing on one mbarrier per stage;
 //   * the warp computes an online softmax over the item's tokens for the G
 //     query heads of the KV head (running max m in log2 units, running sum l,
 //     unnormalised accumulator o, all fp32);
@@ -22,6 +22,8 @@
 // leaves.  Page ids outside the pool are recorded and replaced by page 0.
 #include <math.h>
 
+#include <type_traits>
+
 #include "kvd_internal.h"
 #include "kvd_ptx.cuh"
 
@@ -31,6 +33,7 @@ namespace {
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int kWarps = 4;
+constexpr int kMergeBytes = kMaxChunks * kMaxGroup * 8;   // per-warp (m, l) / weight table
 
 template <int D>
 struct Geo {
@@ -38,7 +41,8 @@ struct Geo {
     static constexpr int kTileBytes = kPageSize * D * 2; // one (page, head) tile
     static constexpr int kStageBytes = 2 * kTileBytes;   // K tile + V tile
     static constexpr int kRing = (D == 128) ? 3 : 6;     // stages per warp
-    static constexpr int kSmem = kWarps * kRing * kStageBytes + kWarps * kRing * 8 + 1024;
+    static constexpr int kRingBytes = kWarps * kRing * kStageBytes;
+    static constexpr int kSmem = kRingBytes + kWarps * kMergeBytes + kWarps * kRing * 8 + 1024;
 };
 
 // Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r, for a tile that
@@ -73,62 +77,385 @@ __device__ __forceinline__ void axpy8(float (&o)[8], float p, const uint4& v)
     o[7] = fmaf(p, bf16hi(v.w), o[7]);
 }
 
-// Merge the partials of (row b, KV head g): one warp, D/32 dims per lane.
-template <int D>
-__device__ void merge_partials(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+// Merge the partials of (row b, KV head g) into the bf16 output rows of its
+// G query heads.  One warp; `wsm` (kMergeBytes of the warp's shared memory)
+// holds the per-(chunk, head) weights.
+//   M_h = max_c m_ch,  w_ch = 2^(m_ch - M_h) / sum_c 2^(m_ch - M_h) l_ch,
+//   O_h = sum_c w_ch o_ch.
+// Loads are issued several chunks at a time so the merge is not bound by
+// one L2 round trip per chunk.
+template <int D, bool GQA>
+__device__ void merge_partials(const DecodeParams& p, const PlanEntry& en, int g, int lane, float* wsm)
 {
-    constexpr int PER = D / 32;
-    const int G = p.G;
-    for (int h = 0; h < G; ++h) {
-        float M = -INFINITY;
-        for (int c = lane; c < en.n_chunks; c += 32) {
-            const float2 ml = __ldcg(&p.part_ml[((int64_t)(en.slot_base + c) * p.H_kv + g) * G + h]);
-            M = fmaxf(M, ml.x);
+    constexpr int PER = D / 32;                 // dims per lane
+    constexpr int HMAX = GQA ? kMaxGroup : 1;
+    constexpr int U = GQA ? 2 : 8;              // chunks in flight per round
+    const int G = GQA ? p.G : 1;
+    const int nch = en.n_chunks;
+    auto slot_of = [&](int c) { return ((int64_t)(en.slot_base + c) * p.H_kv + g) * G; };
+
+    for (int i = lane; i < nch * G; i += 32) {
+        const int c = i / G, h = i - c * G;
+        const float2 ml = __ldcg(&p.part_ml[slot_of(c) + h]);
+        wsm[2 * i] = ml.x;
+        wsm[2 * i + 1] = ml.y;
+    }
+    __syncwarp();
+    {
+        // lanes 4h .. 4h+3 reduce head h over chunks c = lane%4, +4, ...
+        const int h = lane >> 2, q4 = lane & 3;
+        float M = -INFINITY, L = 0.f;
+        if (h < G)
+            for (int c = q4; c < nch; c += 4) M = fmaxf(M, wsm[2 * (c * G + h)]);
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
+        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 2));
+        if (h < G)
+            for (int c = q4; c < nch; c += 4) L = fmaf(ex2(wsm[2 * (c * G + h)] - M), wsm[2 * (c * G + h) + 1], L);
+        L += __shfl_xor_sync(0xffffffffu, L, 1);
+        L += __shfl_xor_sync(0xffffffffu, L, 2);
+        __syncwarp();
+        const float invL = 1.f / L;
+        if (h < G)
+            for (int c = q4; c < nch; c += 4) wsm[2 * (c * G + h)] = ex2(wsm[2 * (c * G + h)] - M) * invL;
+        __syncwarp();
+    }
+    float acc[HMAX][PER];
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h)
+#pragma unroll
+        for (int k = 0; k < PER; ++k) acc[h][k] = 0.f;
+    for (int c0 = 0; c0 < nch; c0 += U) {
+        float v[U][HMAX][PER];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int c = c0 + u;
+#pragma unroll
+            for (int h = 0; h < HMAX; ++h) {
+                if (c < nch && h < G) {
+                    const float* po = p.part_o + (slot_of(c) + h) * D + lane * PER;
+                    if constexpr (PER == 4) {
+                        const float4 t = __ldcg(reinterpret_cast<const float4*>(po));
+                        v[u][h][0] = t.x; v[u][h][1] = t.y; v[u][h][2] = t.z; v[u][h][3] = t.w;
+                    } else {
+                        const float2 t = __ldcg(reinterpret_cast<const float2*>(po));
+                        v[u][h][0] = t.x; v[u][h][1] = t.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int k = 0; k < PER; ++k) v[u][h][k] = 0.f;
+                }
+            }
         }
 #pragma unroll
-        for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-        float L = 0.f, acc[PER];
+        for (int u = 0; u < U; ++u) {
+            const int c = c0 + u;
 #pragma unroll
-        for (int k = 0; k < PER; ++k) acc[k] = 0.f;
-        for (int c = 0; c < en.n_chunks; ++c) {
-            const int64_t slot = ((int64_t)(en.slot_base + c) * p.H_kv + g) * G + h;
-            const float2 ml = __ldcg(&p.part_ml[slot]);
-            const float w = ex2(ml.x - M);
-            L = fmaf(w, ml.y, L);
-            const float* po = p.part_o + slot * D + lane * PER;
+            for (int h = 0; h < HMAX; ++h) {
+                const float w = (c < nch && h < G) ? wsm[2 * (c * G + h)] : 0.f;
 #pragma unroll
-            for (int k = 0; k < PER; ++k) acc[k] = fmaf(w, __ldcg(po + k), acc[k]);
-        }
-        const float inv = 1.f / L;
-        uint16_t* orow = p.out + ((int64_t)en.b * p.H_q + g * G + h) * D + lane * PER;
-        if constexpr (PER == 4) {
-            uint2 v;
-            v.x = pack_bf16(acc[0] * inv, acc[1] * inv);
-            v.y = pack_bf16(acc[2] * inv, acc[3] * inv);
-            *reinterpret_cast<uint2*>(orow) = v;
-        } else {
-            *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0] * inv, acc[1] * inv);
+                for (int k = 0; k < PER; ++k) acc[h][k] = fmaf(w, v[u][h][k], acc[h][k]);
+            }
         }
     }
+#pragma unroll
+    for (int h = 0; h < HMAX; ++h) {
+        if (h < G) {
+            uint16_t* orow = p.out + ((int64_t)en.b * p.H_q + g * G + h) * D + lane * PER;
+            if constexpr (PER == 4) {
+                uint2 o;
+                o.x = pack_bf16(acc[h][0], acc[h][1]);
+                o.y = pack_bf16(acc[h][2], acc[h][3]);
+                *reinterpret_cast<uint2*>(orow) = o;
+            } else {
+                *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[h][0], acc[h][1]);
+            }
+        }
+    }
+    __syncwarp();
 }
 
-// Publish this item's partial and, if it is the row's last, merge.
-template <int D>
-__device__ __forceinline__ void finish_split(const DecodeParams& p, const PlanEntry& en, int g,
-                                             int lane)
+// Take the ticket of a finished split item whose partial the lanes have
+// stored; the warp that takes the row's last ticket merges.  One lane orders
+// the warp's stores before its ticket (the warp barrier makes the other
+// lanes' stores visible to it first); lane 31 is used because lane 0 issues
+// the TMA loads, which a fence in that lane might wait for.
+template <int D, bool GQA>
+__device__ __forceinline__ void take_ticket(const DecodeParams& p, const PlanEntry& en, int g, int lane, float* wsm)
 {
-    __threadfence();
     __syncwarp();
     int last = 0;
     int32_t* ticket = p.tickets + (int64_t)en.b * p.H_kv + g;
-    if (lane == 0) last = (atomicAdd(ticket, 1) == en.n_chunks - 1);
-    last = __shfl_sync(0xffffffffu, last, 0);
+    if (lane == 31) {
+        __threadfence();
+        last = (atomicAdd(ticket, 1) == en.n_chunks - 1);
+    }
+    last = __shfl_sync(0xffffffffu, last, 31);
     if (last) {
         __threadfence();
-        merge_partials<D>(p, en, g, lane);
-        if (lane == 0) *ticket = 0;   // ready for the next layer
+        merge_partials<D, GQA>(p, en, g, lane, wsm);
+        if (lane == 31) *ticket = 0;   // ready for the next layer
     }
 }
+
+// ------------------------------------------------------------ MHA, CUDA cores
+// A lane owns 16-byte chunk c of a row; TPI rows are covered per warp load.
+template <int D>
+struct MhaCompute {
+    static constexpr int CH = D / 8;
+    static constexpr int TPI = 32 / CH;
+    static constexpr int IT = kPageSize / TPI;
+    static constexpr int LOG_IT = (IT == 8) ? 3 : (IT == 4 ? 2 : 1);
+    int c, tsub;
+    float qf[8];
+    float m, l, o[8];
+
+    __device__ __forceinline__ void start(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    {
+        c = lane % CH;
+        tsub = lane / CH;
+        const uint4 qq = *reinterpret_cast<const uint4*>(p.q + ((int64_t)en.b * p.H_q + g) * D + c * 8);
+        qf[0] = bf16lo(qq.x); qf[1] = bf16hi(qq.x);
+        qf[2] = bf16lo(qq.y); qf[3] = bf16hi(qq.y);
+        qf[4] = bf16lo(qq.z); qf[5] = bf16hi(qq.z);
+        qf[6] = bf16lo(qq.w); qf[7] = bf16hi(qq.w);
+        m = -INFINITY;
+        l = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) o[k] = 0.f;
+    }
+
+    __device__ __forceinline__ void page(uint8_t* sK, uint8_t* sV, uint32_t, uint32_t, int valid,
+                                         float scale_log2, int lane)
+    {
+        float part[IT];
+#pragma unroll
+        for (int i = 0; i < IT; ++i) {
+            const uint4 kv = *reinterpret_cast<const uint4*>(sK + swz(i * TPI + tsub, c));
+            part[i] = dot8(kv, qf);
+        }
+        // Reduce-scatter over the CH lanes of a row: afterwards lane c holds
+        // token (c >> 1) * TPI + tsub, summed over all chunks.
+#pragma unroll
+        for (int lv = 0; lv < LOG_IT; ++lv) {
+            const int n = IT >> lv;
+            const int mask = CH >> (lv + 1);
+            const bool hi = (c & mask) != 0;
+#pragma unroll
+            for (int k = 0; k < n / 2; ++k) {
+                const float send = hi ? part[k] : part[k + n / 2];
+                const float keep = hi ? part[k + n / 2] : part[k];
+                part[k] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
+            }
+        }
+        float sc = part[0] + __shfl_xor_sync(0xffffffffu, part[0], 1);
+        const int tok = (c >> 1) * TPI + tsub;
+        sc = (tok < valid) ? sc * scale_log2 : -INFINITY;
+        float pm = sc;
+#pragma unroll
+        for (int mask = 2; mask < 32; mask <<= 1) pm = fmaxf(pm, __shfl_xor_sync(0xffffffffu, pm, mask));
+        const float mn = fmaxf(m, pm);
+        const float alpha = ex2(m - mn);
+        const float pe = ex2(sc - mn);
+        l = fmaf(l, alpha, (c & 1) ? 0.f : pe);
+        m = mn;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) o[k] *= alpha;
+#pragma unroll
+        for (int i = 0; i < IT; ++i) {
+            const float pt = __shfl_sync(0xffffffffu, pe, tsub * CH + 2 * i);
+            const int t = i * TPI + tsub;
+            if (t < valid) {   // rows past the end may hold anything
+                const uint4 vv = *reinterpret_cast<const uint4*>(sV + swz(t, c));
+                axpy8(o, pt, vv);
+            }
+        }
+    }
+
+    // Writes the output (one item) or the partial (split row); returns true
+    // when a partial was stored and the row's ticket is due.
+    __device__ __forceinline__ bool finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    {
+#pragma unroll
+        for (int mask = CH; mask < 32; mask <<= 1)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[k] += __shfl_xor_sync(0xffffffffu, o[k], mask);
+#pragma unroll
+        for (int mask = 1; mask < 32; mask <<= 1) l += __shfl_xor_sync(0xffffffffu, l, mask);
+        if (en.n_chunks == 1) {
+            if (tsub == 0) {
+                const float inv = 1.f / l;
+                uint4 v;
+                v.x = pack_bf16(o[0] * inv, o[1] * inv);
+                v.y = pack_bf16(o[2] * inv, o[3] * inv);
+                v.z = pack_bf16(o[4] * inv, o[5] * inv);
+                v.w = pack_bf16(o[6] * inv, o[7] * inv);
+                *reinterpret_cast<uint4*>(p.out + ((int64_t)en.b * p.H_q + g) * D + c * 8) = v;
+            }
+        } else {
+            const int64_t slot = (int64_t)(en.slot_base + en.chunk) * p.H_kv + g;
+            if (tsub == 0) {
+                float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + c * 8);
+                dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+                dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+            }
+            if (lane == 0) p.part_ml[slot] = make_float2(m, l);
+            return true;
+        }
+        return false;
+    }
+};
+
+// ------------------------------------------------------------ GQA, bf16 MMA
+// S^T[16 tokens][8 heads] = K . q^T and O^T[D][8 heads] += V^T . P^T with
+// mma.m16n8k16; accumulator columns of a lane are heads 2*(lane&3) and +1.
+template <int D>
+struct GqaCompute {
+    static constexpr int KS = D / 16;
+    int G;
+    uint32_t qb[KS][2];
+    float m0, m1, l0, l1;
+    float oacc[KS][4];
+
+    __device__ __forceinline__ void start(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    {
+        G = p.G;
+        const int n = lane >> 2;
+        const uint16_t* qrow = p.q + ((int64_t)en.b * p.H_q + g * G + (n < G ? n : 0)) * D;
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+            const uint32_t x0 = *reinterpret_cast<const uint32_t*>(qrow + ks * 16 + 2 * (lane & 3));
+            const uint32_t x1 = *reinterpret_cast<const uint32_t*>(qrow + ks * 16 + 8 + 2 * (lane & 3));
+            qb[ks][0] = (n < G) ? x0 : 0u;
+            qb[ks][1] = (n < G) ? x1 : 0u;
+        }
+        m0 = m1 = -INFINITY;
+        l0 = l1 = 0.f;
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) oacc[mt][k] = 0.f;
+    }
+
+    __device__ __forceinline__ void page(uint8_t*, uint8_t* sVp, uint32_t sK, uint32_t sV, int valid,
+                                         float scale_log2, int lane)
+    {
+        float sc[4] = {0.f, 0.f, 0.f, 0.f};
+        {
+            const int r = (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+            for (int ks = 0; ks < KS; ++ks) {
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4(sK + swz(r, ks * 2 + (lane >> 4)), a0, a1, a2, a3);
+                mma_bf16_16816(sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+            }
+        }
+        const int t0 = lane >> 2, t1 = t0 + 8;
+        const bool v0 = t0 < valid, v1 = t1 < valid;
+        sc[0] = v0 ? sc[0] * scale_log2 : -INFINITY;
+        sc[1] = v0 ? sc[1] * scale_log2 : -INFINITY;
+        sc[2] = v1 ? sc[2] * scale_log2 : -INFINITY;
+        sc[3] = v1 ? sc[3] * scale_log2 : -INFINITY;
+        float pm0 = fmaxf(sc[0], sc[2]), pm1 = fmaxf(sc[1], sc[3]);
+#pragma unroll
+        for (int mask = 4; mask < 32; mask <<= 1) {
+            pm0 = fmaxf(pm0, __shfl_xor_sync(0xffffffffu, pm0, mask));
+            pm1 = fmaxf(pm1, __shfl_xor_sync(0xffffffffu, pm1, mask));
+        }
+        const float mn0 = fmaxf(m0, pm0), mn1 = fmaxf(m1, pm1);
+        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+        const float p0 = ex2(sc[0] - mn0), p1 = ex2(sc[1] - mn1);
+        const float p2 = ex2(sc[2] - mn0), p3 = ex2(sc[3] - mn1);
+        l0 = fmaf(l0, al0, p0 + p2);
+        l1 = fmaf(l1, al1, p1 + p3);
+        m0 = mn0;
+        m1 = mn1;
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) {
+            oacc[mt][0] *= al0;
+            oacc[mt][1] *= al1;
+            oacc[mt][2] *= al0;
+            oacc[mt][3] *= al1;
+        }
+        // P^T as the B operand: lane needs P[t=2(lane&3)+{0,1}][h=lane>>2] and
+        // the same for t+8.  P[t][h] for t < 8 sits in lane 4t + h/2.
+        const int srcA = 8 * (lane & 3) + (lane >> 3);
+        const int srcB = srcA + 4;
+        const uint32_t u01 = pack_bf16(p0, p1), u23 = pack_bf16(p2, p3);
+        const uint32_t xa = __shfl_sync(0xffffffffu, u01, srcA);
+        const uint32_t xb = __shfl_sync(0xffffffffu, u01, srcB);
+        const uint32_t za = __shfl_sync(0xffffffffu, u23, srcA);
+        const uint32_t zb = __shfl_sync(0xffffffffu, u23, srcB);
+        const uint32_t sel = ((lane >> 2) & 1) ? 0x7632u : 0x5410u;
+        const uint32_t pb0 = __byte_perm(xa, xb, sel);
+        const uint32_t pb1 = __byte_perm(za, zb, sel);
+
+        if (valid < kPageSize) {   // rows past the end may hold anything
+            constexpr int CH = D / 8;
+            for (int i = lane; i < (kPageSize - valid) * CH; i += 32) {
+                const int r = valid + i / CH;
+                *reinterpret_cast<uint4*>(sVp + swz(r, i % CH)) = make_uint4(0, 0, 0, 0);
+            }
+            __syncwarp();
+        }
+        {
+            const int r = (lane & 7) + (lane >> 4) * 8;
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4_trans(sV + swz(r, mt * 2 + ((lane >> 3) & 1)), a0, a1, a2, a3);
+                mma_bf16_16816(oacc[mt], a0, a1, a2, a3, pb0, pb1);
+            }
+        }
+    }
+
+    __device__ __forceinline__ bool finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    {
+#pragma unroll
+        for (int mask = 4; mask < 32; mask <<= 1) {
+            l0 += __shfl_xor_sync(0xffffffffu, l0, mask);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, mask);
+        }
+        const int h0 = 2 * (lane & 3), h1 = h0 + 1;
+        const int dlo = lane >> 2;
+        if (en.n_chunks == 1) {
+            const float i0 = 1.f / l0, i1 = 1.f / l1;
+            uint16_t* ob = p.out + ((int64_t)en.b * p.H_q + g * G) * D;
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                const int d0 = mt * 16 + dlo;
+                if (h0 < G) {
+                    ob[h0 * D + d0] = (uint16_t)(pack_bf16(oacc[mt][0] * i0, 0.f) & 0xffffu);
+                    ob[h0 * D + d0 + 8] = (uint16_t)(pack_bf16(oacc[mt][2] * i0, 0.f) & 0xffffu);
+                }
+                if (h1 < G) {
+                    ob[h1 * D + d0] = (uint16_t)(pack_bf16(oacc[mt][1] * i1, 0.f) & 0xffffu);
+                    ob[h1 * D + d0 + 8] = (uint16_t)(pack_bf16(oacc[mt][3] * i1, 0.f) & 0xffffu);
+                }
+            }
+        } else {
+            const int64_t slot = (int64_t)(en.slot_base + en.chunk) * p.H_kv + g;
+            float* po = p.part_o + slot * G * D;
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+                const int d0 = mt * 16 + dlo;
+                if (h0 < G) {
+                    po[h0 * D + d0] = oacc[mt][0];
+                    po[h0 * D + d0 + 8] = oacc[mt][2];
+                }
+                if (h1 < G) {
+                    po[h1 * D + d0] = oacc[mt][1];
+                    po[h1 * D + d0 + 8] = oacc[mt][3];
+                }
+            }
+            if (lane < 4) {
+                if (h0 < G) p.part_ml[slot * G + h0] = make_float2(m0, l0);
+                if (h1 < G) p.part_ml[slot * G + h1] = make_float2(m1, l1);
+            }
+            return true;
+        }
+        return false;
+    }
+};
 
 template <int D, bool GQA>
 __global__ void __launch_bounds__(kWarps * 32)
@@ -145,7 +472,8 @@ __global__ void __launch_bounds__(kWarps * 32)
                                                ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t* ring = smem + warp * R * STAGE;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * R * STAGE) + warp * R;
+    float* wsm = reinterpret_cast<float*>(smem + Gm::kRingBytes + warp * kMergeBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Gm::kRingBytes + kWarps * kMergeBytes) + warp * R;
     const uint32_t ring_s = smem_addr(ring);
 
     if (lane == 0) {
@@ -164,30 +492,37 @@ __global__ void __launch_bounds__(kWarps * 32)
     uint32_t pending = 0;  // bit s: stage s has a load in flight that was not waited on
     bool ok = true;
 
-    while (ok) {
-        int item = 0;
-        if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
-        item = __shfl_sync(0xffffffffu, item, 0);
-        if (item >= p.n_items) break;
+    using Comp = typename std::conditional<GQA, GqaCompute<D>, MhaCompute<D>>::type;
+    Comp comp;
+
+    int item = 0;
+    if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
+    item = __shfl_sync(0xffffffffu, item, 0);
+
+    while (item < p.n_items) {
         const int e = item / p.H_kv;
         const int g = item - e * p.H_kv;
         const PlanEntry en = p.plan[e];
         const int np = en.n_pages;
 
-        // Page ids of the item: lane j holds pages j and j + 32.
+        // Page ids of the item in windows of 32: lane i holds page w*32 + i of
+        // the current window; the next window is fetched 24 pages ahead.
         const int32_t* pt_row = p.page_table + (int64_t)en.seq * p.max_pages + en.first_page;
-        int32_t pid0 = (lane < np) ? pt_row[lane] : 0;
-        int32_t pid1 = (lane + 32 < np) ? pt_row[lane + 32] : 0;
-        const bool bad = (pid0 < 0 || pid0 >= p.num_pages) || (pid1 < 0 || pid1 >= p.num_pages);
-        if (bad) {
-            atomicOr(p.err, 1);
-            if (pid0 < 0 || pid0 >= p.num_pages) pid0 = 0;
-            if (pid1 < 0 || pid1 >= p.num_pages) pid1 = 0;
-        }
+        auto load_window = [&](int w0) {
+            int32_t v = (w0 + lane < np) ? pt_row[w0 + lane] : 0;
+            if (v < 0 || v >= p.num_pages) {
+                atomicOr(p.err, 1);
+                v = 0;
+            }
+            return v;
+        };
+        int32_t pid_cur = load_window(0);
+        int32_t pid_next = 0;
 
         auto issue = [&](int j, int s) {
-            const int32_t pid = (j < 32) ? __shfl_sync(0xffffffffu, pid0, j & 31)
-                                         : __shfl_sync(0xffffffffu, pid1, j & 31);
+            if ((j & 31) == 8 && j + 24 < np) pid_next = load_window(j + 24);
+            if ((j & 31) == 0 && j > 0) pid_cur = pid_next;
+            const int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
             if (lane == 0) {
                 const uint32_t bar = smem_addr(&bars[s]);
                 const uint32_t dst = ring_s + s * STAGE;
@@ -206,272 +541,33 @@ __global__ void __launch_bounds__(kWarps * 32)
         __syncwarp();
         for (int j = 0; j < pre; ++j) issue(j, j);
         pending = (1u << pre) - 1u;
+        comp.start(p, en, g, lane);
 
-        if constexpr (!GQA) {
-            // ------------------------------------------------ MHA, CUDA cores
-            constexpr int CH = D / 8;          // 16-byte chunks per row
-            constexpr int TPI = 32 / CH;       // tokens covered by one warp load
-            constexpr int IT = kPageSize / TPI;
-            constexpr int LOG_IT = (IT == 8) ? 3 : (IT == 4 ? 2 : 1);
-            const int c = lane % CH, tsub = lane / CH;
-            float qf[8];
-            {
-                const uint4 qq = *reinterpret_cast<const uint4*>(
-                    p.q + ((int64_t)en.b * p.H_q + g) * D + c * 8);
-                qf[0] = bf16lo(qq.x); qf[1] = bf16hi(qq.x);
-                qf[2] = bf16lo(qq.y); qf[3] = bf16hi(qq.y);
-                qf[4] = bf16lo(qq.z); qf[5] = bf16hi(qq.z);
-                qf[6] = bf16lo(qq.w); qf[7] = bf16hi(qq.w);
+        for (int j = 0; j < np; ++j) {
+            const int s = j % R;
+            const bool w = mbar_wait_bounded(smem_addr(&bars[s]), (phase >> s) & 1u, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, w)) {
+                ok = false;
+                break;
             }
-            float m = -INFINITY, l = 0.f, o[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) o[k] = 0.f;
-
-            for (int j = 0; j < np; ++j) {
-                const int s = j % R;
-                const bool w = mbar_wait_bounded(smem_addr(&bars[s]), (phase >> s) & 1u, kWaitLimitNs);
-                if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
-                phase ^= 1u << s;
-                pending &= ~(1u << s);
-                const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
-                const uint8_t* sK = ring + s * STAGE;
-                const uint8_t* sV = sK + TILE;
-
-                float part[IT];
-#pragma unroll
-                for (int i = 0; i < IT; ++i) {
-                    const uint4 kv = *reinterpret_cast<const uint4*>(sK + swz(i * TPI + tsub, c));
-                    part[i] = dot8(kv, qf);
-                }
-                // Reduce-scatter over the CH lanes of a row: afterwards lane c
-                // holds token (c >> 1) * TPI + tsub, summed over all chunks.
-#pragma unroll
-                for (int lv = 0; lv < LOG_IT; ++lv) {
-                    const int n = IT >> lv;
-                    const int mask = CH >> (lv + 1);
-                    const bool hi = (c & mask) != 0;
-#pragma unroll
-                    for (int k = 0; k < n / 2; ++k) {
-                        const float send = hi ? part[k] : part[k + n / 2];
-                        const float keep = hi ? part[k + n / 2] : part[k];
-                        part[k] = keep + __shfl_xor_sync(0xffffffffu, send, mask);
-                    }
-                }
-                float sc = part[0] + __shfl_xor_sync(0xffffffffu, part[0], 1);
-                const int tok = (c >> 1) * TPI + tsub;
-                sc = (tok < valid) ? sc * p.scale_log2 : -INFINITY;
-                float pm = sc;
-#pragma unroll
-                for (int mask = 2; mask < 32; mask <<= 1)
-                    pm = fmaxf(pm, __shfl_xor_sync(0xffffffffu, pm, mask));
-                const float mn = fmaxf(m, pm);
-                const float alpha = ex2(m - mn);
-                const float pe = ex2(sc - mn);
-                l = fmaf(l, alpha, (c & 1) ? 0.f : pe);
-                m = mn;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) o[k] *= alpha;
-#pragma unroll
-                for (int i = 0; i < IT; ++i) {
-                    const float pt = __shfl_sync(0xffffffffu, pe, tsub * CH + 2 * i);
-                    const int t = i * TPI + tsub;
-                    if (t < valid) {
-                        const uint4 vv = *reinterpret_cast<const uint4*>(sV + swz(t, c));
-                        axpy8(o, pt, vv);
-                    }
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (j + R < np) {
-                    issue(j + R, s);
-                    pending |= 1u << s;
-                }
-            }
-            if (!ok) break;
-#pragma unroll
-            for (int mask = CH; mask < 32; mask <<= 1)
-#pragma unroll
-                for (int k = 0; k < 8; ++k) o[k] += __shfl_xor_sync(0xffffffffu, o[k], mask);
-#pragma unroll
-            for (int mask = 1; mask < 32; mask <<= 1) l += __shfl_xor_sync(0xffffffffu, l, mask);
-
-            if (en.n_chunks == 1) {
-                if (tsub == 0) {
-                    const float inv = 1.f / l;
-                    uint4 v;
-                    v.x = pack_bf16(o[0] * inv, o[1] * inv);
-                    v.y = pack_bf16(o[2] * inv, o[3] * inv);
-                    v.z = pack_bf16(o[4] * inv, o[5] * inv);
-                    v.w = pack_bf16(o[6] * inv, o[7] * inv);
-                    *reinterpret_cast<uint4*>(p.out + ((int64_t)en.b * p.H_q + g) * D + c * 8) = v;
-                }
-            } else {
-                const int64_t slot = (int64_t)(en.slot_base + en.chunk) * p.H_kv + g;
-                if (tsub == 0) {
-                    float4* dst = reinterpret_cast<float4*>(p.part_o + slot * D + c * 8);
-                    dst[0] = make_float4(o[0], o[1], o[2], o[3]);
-                    dst[1] = make_float4(o[4], o[5], o[6], o[7]);
-                }
-                if (lane == 0) p.part_ml[slot] = make_float2(m, l);
-                finish_split<D>(p, en, g, lane);
-            }
-        } else {
-            // ------------------------------------------------ GQA, bf16 MMA
-            constexpr int KS = D / 16;
-            const int G = p.G;
-            const int n = lane >> 2;           // head of this lane's B-fragment column
-            uint32_t qb[KS][2];
-            {
-                const uint16_t* qrow = p.q + ((int64_t)en.b * p.H_q + g * G + (n < G ? n : 0)) * D;
-#pragma unroll
-                for (int ks = 0; ks < KS; ++ks) {
-                    uint32_t x0 = *reinterpret_cast<const uint32_t*>(qrow + ks * 16 + 2 * (lane & 3));
-                    uint32_t x1 = *reinterpret_cast<const uint32_t*>(qrow + ks * 16 + 8 + 2 * (lane & 3));
-                    qb[ks][0] = (n < G) ? x0 : 0u;
-                    qb[ks][1] = (n < G) ? x1 : 0u;
-                }
-            }
-            // Accumulator columns of this lane: heads h0 = 2*(lane&3), h1 = h0+1.
-            float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-            float oacc[KS][4];
-#pragma unroll
-            for (int mt = 0; mt < KS; ++mt)
-#pragma unroll
-                for (int k = 0; k < 4; ++k) oacc[mt][k] = 0.f;
-            const int t0 = lane >> 2, t1 = t0 + 8;
-            const int srcA = 8 * (lane & 3) + (lane >> 3);
-            const int srcB = srcA + 4;
-            const bool hodd = (n & 1) != 0;
-
-            for (int j = 0; j < np; ++j) {
-                const int s = j % R;
-                const bool w = mbar_wait_bounded(smem_addr(&bars[s]), (phase >> s) & 1u, kWaitLimitNs);
-                if (!__all_sync(0xffffffffu, w)) { ok = false; break; }
-                phase ^= 1u << s;
-                pending &= ~(1u << s);
-                const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
-                const uint32_t sK = ring_s + s * STAGE;
-                const uint32_t sV = sK + TILE;
-
-                // S^T[16 tokens][8 heads] = K . q^T
-                float sc[4] = {0.f, 0.f, 0.f, 0.f};
-                {
-                    const int r = (lane & 7) + ((lane >> 3) & 1) * 8;
-#pragma unroll
-                    for (int ks = 0; ks < KS; ++ks) {
-                        uint32_t a0, a1, a2, a3;
-                        ldsm_x4(sK + swz(r, ks * 2 + (lane >> 4)), a0, a1, a2, a3);
-                        mma_bf16_16816(sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
-                    }
-                }
-                const bool v0 = t0 < valid, v1 = t1 < valid;
-                sc[0] = v0 ? sc[0] * p.scale_log2 : -INFINITY;
-                sc[1] = v0 ? sc[1] * p.scale_log2 : -INFINITY;
-                sc[2] = v1 ? sc[2] * p.scale_log2 : -INFINITY;
-                sc[3] = v1 ? sc[3] * p.scale_log2 : -INFINITY;
-                float pm0 = fmaxf(sc[0], sc[2]), pm1 = fmaxf(sc[1], sc[3]);
-#pragma unroll
-                for (int mask = 4; mask < 32; mask <<= 1) {
-                    pm0 = fmaxf(pm0, __shfl_xor_sync(0xffffffffu, pm0, mask));
-                    pm1 = fmaxf(pm1, __shfl_xor_sync(0xffffffffu, pm1, mask));
-                }
-                const float mn0 = fmaxf(m0, pm0), mn1 = fmaxf(m1, pm1);
-                const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
-                const float p0 = ex2(sc[0] - mn0), p1 = ex2(sc[1] - mn1);
-                const float p2 = ex2(sc[2] - mn0), p3 = ex2(sc[3] - mn1);
-                l0 = fmaf(l0, al0, p0 + p2);
-                l1 = fmaf(l1, al1, p1 + p3);
-                m0 = mn0;
-                m1 = mn1;
-#pragma unroll
-                for (int mt = 0; mt < KS; ++mt) {
-                    oacc[mt][0] *= al0;
-                    oacc[mt][1] *= al1;
-                    oacc[mt][2] *= al0;
-                    oacc[mt][3] *= al1;
-                }
-                // P^T as the B operand: lane needs P[t=2(lane&3)+{0,1}][h=lane>>2]
-                // and the same for t+8.
-                const uint32_t u01 = pack_bf16(p0, p1), u23 = pack_bf16(p2, p3);
-                const uint32_t xa = __shfl_sync(0xffffffffu, u01, srcA);
-                const uint32_t xb = __shfl_sync(0xffffffffu, u01, srcB);
-                const uint32_t za = __shfl_sync(0xffffffffu, u23, srcA);
-                const uint32_t zb = __shfl_sync(0xffffffffu, u23, srcB);
-                const uint32_t sel = hodd ? 0x7632u : 0x5410u;
-                const uint32_t pb0 = __byte_perm(xa, xb, sel);
-                const uint32_t pb1 = __byte_perm(za, zb, sel);
-
-                if (valid < kPageSize) {   // rows past the end may hold anything
-                    constexpr int CH = D / 8;
-                    uint8_t* sVp = ring + s * STAGE + TILE;
-                    for (int i = lane; i < (kPageSize - valid) * CH; i += 32) {
-                        const int r = valid + i / CH;
-                        *reinterpret_cast<uint4*>(sVp + swz(r, i % CH)) = make_uint4(0, 0, 0, 0);
-                    }
-                    __syncwarp();
-                }
-                // O^T[D][8 heads] += V^T . P^T
-                {
-                    const int r = (lane & 7) + (lane >> 4) * 8;
-#pragma unroll
-                    for (int mt = 0; mt < KS; ++mt) {
-                        uint32_t a0, a1, a2, a3;
-                        ldsm_x4_trans(sV + swz(r, mt * 2 + ((lane >> 3) & 1)), a0, a1, a2, a3);
-                        mma_bf16_16816(oacc[mt], a0, a1, a2, a3, pb0, pb1);
-                    }
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (j + R < np) {
-                    issue(j + R, s);
-                    pending |= 1u << s;
-                }
-            }
-            if (!ok) break;
-#pragma unroll
-            for (int mask = 4; mask < 32; mask <<= 1) {
-                l0 += __shfl_xor_sync(0xffffffffu, l0, mask);
-                l1 += __shfl_xor_sync(0xffffffffu, l1, mask);
-            }
-            const int h0 = 2 * (lane & 3), h1 = h0 + 1;
-            const int dlo = lane >> 2;
-            if (en.n_chunks == 1) {
-                const float i0 = 1.f / l0, i1 = 1.f / l1;
-                uint16_t* ob = p.out + ((int64_t)en.b * p.H_q + g * G) * D;
-#pragma unroll
-                for (int mt = 0; mt < KS; ++mt) {
-                    const int d0 = mt * 16 + dlo;
-                    if (h0 < G) {
-                        ob[h0 * D + d0] = (uint16_t)(pack_bf16(oacc[mt][0] * i0, 0.f) & 0xffffu);
-                        ob[h0 * D + d0 + 8] = (uint16_t)(pack_bf16(oacc[mt][2] * i0, 0.f) & 0xffffu);
-                    }
-                    if (h1 < G) {
-                        ob[h1 * D + d0] = (uint16_t)(pack_bf16(oacc[mt][1] * i1, 0.f) & 0xffffu);
-                        ob[h1 * D + d0 + 8] = (uint16_t)(pack_bf16(oacc[mt][3] * i1, 0.f) & 0xffffu);
-                    }
-                }
-            } else {
-                const int64_t slot = (int64_t)(en.slot_base + en.chunk) * p.H_kv + g;
-                float* po = p.part_o + slot * G * D;
-#pragma unroll
-                for (int mt = 0; mt < KS; ++mt) {
-                    const int d0 = mt * 16 + dlo;
-                    if (h0 < G) {
-                        po[h0 * D + d0] = oacc[mt][0];
-                        po[h0 * D + d0 + 8] = oacc[mt][2];
-                    }
-                    if (h1 < G) {
-                        po[h1 * D + d0] = oacc[mt][1];
-                        po[h1 * D + d0 + 8] = oacc[mt][3];
-                    }
-                }
-                if (lane < 4) {
-                    if (h0 < G) p.part_ml[slot * G + h0] = make_float2(m0, l0);
-                    if (h1 < G) p.part_ml[slot * G + h1] = make_float2(m1, l1);
-                }
-                finish_split<D>(p, en, g, lane);
+            phase ^= 1u << s;
+            pending &= ~(1u << s);
+            const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
+            uint8_t* sK = ring + s * STAGE;
+            comp.page(sK, sK + TILE, ring_s + s * STAGE, ring_s + s * STAGE + TILE, valid, p.scale_log2, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (j + R < np) {
+                issue(j + R, s);
+                pending |= 1u << s;
             }
         }
+        if (!ok) break;
+        // Taking the ticket right away measured faster than deferring it
+        // behind the next item's first loads.
+        if (comp.finish(p, en, g, lane)) take_ticket<D, GQA>(p, en, g, lane, wsm);
+        if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
+        item = __shfl_sync(0xffffffffu, item, 0);
     }
 
     if (!ok && lane == 0) atomicOr(p.err, 2);
@@ -482,8 +578,8 @@ __global__ void __launch_bounds__(kWarps * 32)
     __syncwarp();
 
     // The last warp out resets the work counter for the next launch.
-    __threadfence();
-    if (lane == 0) {
+    if (lane == 31) {
+        __threadfence();
         const uint32_t total = gridDim.x * kWarps;
         if (atomicAdd(&p.queue[1], 1u) == total - 1) {
             p.queue[0] = 0;

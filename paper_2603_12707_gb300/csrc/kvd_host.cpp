@@ -138,14 +138,15 @@ int push_updates(kv_cache* c, const std::vector<int32_t>& idx, const std::vector
     return KVC_OK;
 }
 
-int32_t auto_split_pages(const kv_cache* c, int64_t total_units)
+int32_t auto_item_pages(const kv_cache* c, int64_t total_units)
 {
-    // Aim for about four work items per resident warp so the tail of the
-    // persistent schedule stays short, within [2, kMaxSplitPages] pages.
+    // About three work items per resident warp keeps the tail of the
+    // persistent schedule short; items stay within [2, 128] pages (long rows
+    // get larger items through the per-row cap on the number of items).
     const int64_t warps = (int64_t)std::max(1, c->num_sms) * std::max(1, c->variant.ctas_per_sm) *
                           std::max(1, c->variant.warps);
-    int64_t C = (total_units + 4 * warps - 1) / (4 * warps);
-    return (int32_t)std::min<int64_t>(kMaxSplitPages, std::max<int64_t>(2, C));
+    const int64_t T = (total_units + 3 * warps - 1) / (3 * warps);
+    return (int32_t)std::min<int64_t>(128, std::max<int64_t>(2, T));
 }
 
 int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, cudaStream_t st)
@@ -348,8 +349,8 @@ int kv_cache_pool(kv_cache* c, int32_t layer, void** k_pool, void** v_pool)
 int kv_cache_set_split_pages(kv_cache* c, int32_t pages)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_cache_set_split_pages: null cache");
-    if (pages < 0 || pages > kMaxSplitPages)
-        return fail(KVC_ERR_INVALID, "kv_cache_set_split_pages: pages must be in 0 .. 64");
+    if (pages < 0 || pages > kMaxItemPages)
+        return fail(KVC_ERR_INVALID, "kv_cache_set_split_pages: pages must be in 0 .. 1024");
     c->split_override = pages;
     return KVC_OK;
 }
@@ -489,16 +490,15 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     if (need > (int64_t)c->free_stack.size()) return fail(KVC_ERR_OOM, "kv_begin_step: page pool exhausted");
 
     // Size the plan from the lengths after this step, before changing anything.
+    std::vector<int32_t> np_after((size_t)batch);
     int64_t total_units = 0;
-    for (int32_t b = 0; b < batch; ++b)
-        total_units += (int64_t)((c->lens[seq_ids[b]] + 1 + kPageSize - 1) / kPageSize) * c->cfg.num_kv_heads;
-    const int32_t C = c->split_override ? c->split_override : auto_split_pages(c, total_units);
-    int64_t entries = 0, total_full = 0;
     for (int32_t b = 0; b < batch; ++b) {
-        const int64_t np = (c->lens[seq_ids[b]] + 1 + kPageSize - 1) / kPageSize;
-        total_full += np / C;
-        entries += np / C + (np % C ? 1 : 0);
+        np_after[b] = (c->lens[seq_ids[b]] + 1 + kPageSize - 1) / kPageSize;
+        total_units += (int64_t)np_after[b] * c->cfg.num_kv_heads;
     }
+    const int32_t T = c->split_override ? c->split_override : auto_item_pages(c, total_units);
+    int64_t entries = 0;
+    for (int32_t b = 0; b < batch; ++b) entries += row_chunks(np_after[b], T);
     if (!c->host_only)
         if (int rc = grow_scratch(c, entries, entries * c->cfg.num_kv_heads, static_cast<cudaStream_t>(stream)))
             return rc;
@@ -519,13 +519,20 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         StepPatch patch;
         PlanArgs pa;
         pa.batch = batch;
-        pa.chunk_pages = C;
+        pa.item_pages = T;
         pa.max_pages = c->cfg.max_pages_per_seq;
         pa.step_seq = c->step_seq;
         pa.seq_len = c->seq_len_dev();
         pa.page_table = c->page_table();
         pa.plan = c->plan;
         pa.err = c->err;
+        // Longest rows first: their items start early and the tail is short.
+        pa.use_order = batch <= kPatchMax ? 1 : 0;
+        if (pa.use_order) {
+            for (int32_t b = 0; b < batch; ++b) pa.order[b] = b;
+            std::stable_sort(pa.order, pa.order + batch,
+                             [&](int32_t x, int32_t y) { return np_after[x] > np_after[y]; });
+        }
         for (int32_t b0 = 0; b0 < batch; b0 += kPatchMax) {
             const int32_t n = std::min(kPatchMax, batch - b0);
             patch.n = n;
@@ -536,7 +543,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
                 patch.new_page[i] = new_page[b0 + i];
             }
             pa.build = (b0 + n == batch) ? 1 : 0;
-            KVD_CUDA(launch_step(patch, pa, (int32_t)total_full, st));
+            KVD_CUDA(launch_step(patch, pa, st));
         }
     }
     c->step_active = true;

@@ -10,7 +10,8 @@ namespace kvd {
 
 constexpr int kPageSize = 16;          // tokens per page (the only supported P)
 constexpr int kMaxGroup = 8;           // query heads per KV head handled by one MMA N-tile
-constexpr int kMaxSplitPages = 64;     // pages per work item (two page-id registers per lane)
+constexpr int kMaxChunks = 32;         // work items per (row, KV head) at most
+constexpr int kMaxItemPages = 1024;    // largest target item size a caller may request
 constexpr int kPatchMax = 1024;        // step entries carried in one launch's parameters
 constexpr int kScatterMax = 2048;      // int32 updates carried in one launch's parameters
 
@@ -22,11 +23,29 @@ struct PlanEntry {
     int32_t seq;        // sequence id (page-table row)
     int32_t len;        // tokens attended, including this step's token
     int32_t first_page; // first logical page of the item
-    int32_t n_pages;    // pages of the item, 1 .. kMaxSplitPages
+    int32_t n_pages;    // pages of the item (>= 1)
     int32_t chunk;      // index of the item among the row's items
     int32_t n_chunks;   // items of the row
     int32_t slot_base;  // first partial slot of the row; slot = (slot_base + chunk) * H_kv + g
 };
+
+// Split policy shared by host and device.  A row of np pages is cut into
+// nch items of near-equal size: the target size T, raised for long rows so a
+// row never has more than kMaxChunks items (which bounds the merge).
+__host__ __device__ inline int row_chunks(int np, int T)
+{
+    const int t_row = (np + kMaxChunks - 1) / kMaxChunks;
+    const int Tb = T > t_row ? T : t_row;
+    return (np + Tb - 1) / Tb;
+}
+
+// Pages [first, first + n) of item c of nch over np pages.
+__host__ __device__ inline void chunk_range(int np, int nch, int c, int* first, int* n)
+{
+    const int base = np / nch, extra = np % nch;
+    *first = c * base + (c < extra ? c : extra);
+    *n = base + (c < extra ? 1 : 0);
+}
 
 // Per-step update, passed by value in kernel parameters.
 struct StepPatch {
@@ -40,8 +59,10 @@ struct StepPatch {
 struct PlanArgs {
     int32_t build;       // build the plan in this launch (last launch of a step)
     int32_t batch;
-    int32_t chunk_pages; // C
+    int32_t item_pages;  // target pages per work item (T)
     int32_t max_pages;   // page-table row length
+    int32_t use_order;   // rows are planned in order[] (else batch order)
+    int32_t order[kPatchMax];
     int32_t* step_seq;   // [max_seqs] batch row -> sequence id
     int32_t* seq_len;    // [max_seqs]
     int32_t* page_table; // [max_seqs][max_pages]
@@ -102,9 +123,7 @@ void set_last_error(const char* msg);
 
 // ---- launchers (return cudaGetLastError() of the launch) -----------------
 cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st);
-// total_full: number of full-size items of the plan (the host knows it).
-cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, int32_t total_full,
-                        cudaStream_t st);
+cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, cudaStream_t st);
 cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
 

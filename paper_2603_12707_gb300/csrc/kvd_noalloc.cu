@@ -39,23 +39,22 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes]
 
 struct NoAllocPlanArgs {
     int32_t batch;
-    int32_t chunk_pages;
-    int32_t total_full;
     int32_t n_tickets;     // batch * H_kv
     PlanEntry* plan;
     int32_t* tickets;
     uint32_t* queue;
     int32_t* err;
     int32_t clear_err;
-    int32_t len[kNoAllocMaxBatch];       // tokens attended per row
-    int32_t full_off[kNoAllocMaxBatch];  // first full-size item of the row
-    int32_t rem_off[kNoAllocMaxBatch];   // index of the row's shorter last item (if any)
-    int32_t slot[kNoAllocMaxBatch];      // first partial slot of the row
+    // rows in planning order (longest first)
+    int32_t row[kNoAllocMaxBatch];   // batch row
+    int32_t len[kNoAllocMaxBatch];   // tokens attended
+    int32_t off[kNoAllocMaxBatch];   // first plan entry of the row
+    int32_t nch[kNoAllocMaxBatch];   // items of the row
+    int32_t slot[kNoAllocMaxBatch];  // first partial slot (rows with one item use none)
 };
 
 // One block: clear the tickets and work counters, then write each row's
-// items of C pages (full items first, then every row's shorter last item) at
-// the offsets the host computed.
+// items (near-equal page ranges) at the offsets the host computed.
 __global__ void __launch_bounds__(1024) noalloc_plan_kernel(const __grid_constant__ NoAllocPlanArgs a)
 {
     for (int i = threadIdx.x; i < a.n_tickets; i += blockDim.x) a.tickets[i] = 0;
@@ -64,13 +63,13 @@ __global__ void __launch_bounds__(1024) noalloc_plan_kernel(const __grid_constan
         a.queue[1] = 0;
         if (a.clear_err) *a.err = 0;
     }
-    const int C = a.chunk_pages;
-    for (int b = threadIdx.x; b < a.batch; b += blockDim.x) {
-        const int np = (a.len[b] + kPageSize - 1) / kPageSize;
-        const int full = np / C, rem = (np % C) ? 1 : 0, nch = full + rem;
-        for (int c = 0; c < full; ++c)
-            a.plan[a.full_off[b] + c] = PlanEntry{b, b, a.len[b], c * C, C, c, nch, a.slot[b]};
-        if (rem) a.plan[a.rem_off[b]] = PlanEntry{b, b, a.len[b], full * C, np - full * C, full, nch, a.slot[b]};
+    for (int i = threadIdx.x; i < a.batch; i += blockDim.x) {
+        const int np = (a.len[i] + kPageSize - 1) / kPageSize;
+        for (int c = 0; c < a.nch[i]; ++c) {
+            int first, n;
+            chunk_range(np, a.nch[i], c, &first, &n);
+            a.plan[a.off[i] + c] = PlanEntry{a.row[i], a.row[i], a.len[i], first, n, c, a.nch[i], a.slot[i]};
+        }
     }
 }
 
@@ -168,33 +167,28 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     uint8_t* scratch = nullptr;
     if (int rc = scratch_address(&scratch)) return rc;
 
-    // Split size: the library's usual target (about four items per resident
-    // warp), enlarged until the plan and partials fit the static scratch.
+    // Items: the library's usual target (about three per resident warp),
+    // enlarged until the plan and the partials fit the static scratch.
     const int64_t warps = (int64_t)num_sms * std::max(1, var.ctas_per_sm) * std::max(1, var.warps);
-    int64_t C = std::min<int64_t>(kMaxSplitPages,
-                                  std::max<int64_t>(2, (total_pages * num_kv_heads + 4 * warps - 1) / (4 * warps)));
-    int64_t entries = 0, total_full = 0;
-    size_t off_plan = 0, off_o = 0, off_ml = 0, off_tk = 0, off_q = 0, off_err = 0, need = 0;
-    for (;; C = std::min<int64_t>(kMaxSplitPages, C * 2)) {
+    int64_t T = std::min<int64_t>(128, std::max<int64_t>(2, (total_pages * num_kv_heads + 3 * warps - 1) / (3 * warps)));
+    int64_t entries = 0;
+    size_t off_o = 0, off_ml = 0, off_tk = 0, off_q = 0, off_err = 0, need = 0;
+    for (;; T *= 2) {
         entries = 0;
-        total_full = 0;
         int64_t split_items = 0;   // only rows cut into several items keep partials
         for (int b = 0; b < batch; ++b) {
-            const int64_t np = (lens[b] + kPageSize - 1) / kPageSize;
-            const int64_t nch = np / C + (np % C ? 1 : 0);
-            total_full += np / C;
+            const int64_t nch = row_chunks((lens[b] + kPageSize - 1) / kPageSize, (int)T);
             entries += nch;
             if (nch > 1) split_items += nch;
         }
         const int64_t slots = split_items * num_kv_heads;
-        off_plan = 0;
-        off_o = round256(off_plan + (size_t)entries * sizeof(PlanEntry));
+        off_o = round256((size_t)entries * sizeof(PlanEntry));
         off_ml = round256(off_o + (size_t)slots * G * head_dim * sizeof(float));
         off_tk = round256(off_ml + (size_t)slots * G * sizeof(float2));
         off_q = round256(off_tk + (size_t)batch * num_kv_heads * sizeof(int32_t));
         off_err = off_q + 2 * sizeof(uint32_t);
         need = round256(off_err + sizeof(int32_t));
-        if (need <= kNoAllocScratchBytes || C == kMaxSplitPages) break;
+        if (need <= kNoAllocScratchBytes || T >= kMaxItemPages) break;
     }
     if (need > kNoAllocScratchBytes)
         return fail(KVC_ERR_UNSUPPORTED, ("the batch needs " + std::to_string(need) +
@@ -216,26 +210,25 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
 
     NoAllocPlanArgs pa;
     pa.batch = batch;
-    pa.chunk_pages = (int32_t)C;
-    pa.total_full = (int32_t)total_full;
     pa.n_tickets = batch * num_kv_heads;
-    pa.plan = reinterpret_cast<PlanEntry*>(scratch + off_plan);
+    pa.plan = reinterpret_cast<PlanEntry*>(scratch);
     pa.tickets = reinterpret_cast<int32_t*>(scratch + off_tk);
     pa.queue = reinterpret_cast<uint32_t*>(scratch + off_q);
     pa.err = device_error ? device_error : reinterpret_cast<int32_t*>(scratch + off_err);
     pa.clear_err = device_error ? 0 : 1;
     {
-        int32_t full_off = 0, rem_off = (int32_t)total_full, slot = 0;
-        for (int b = 0; b < batch; ++b) {
-            const int32_t np = (lens[b] + kPageSize - 1) / kPageSize;
-            const int32_t full = np / (int32_t)C, rem = (np % C) ? 1 : 0;
-            pa.len[b] = lens[b];
-            pa.full_off[b] = full_off;
-            pa.rem_off[b] = rem_off;
-            pa.slot[b] = slot;
-            full_off += full;
-            rem_off += rem;
-            if (full + rem > 1) slot += full + rem;
+        for (int b = 0; b < batch; ++b) pa.row[b] = b;
+        std::stable_sort(pa.row, pa.row + batch, [&](int32_t x, int32_t y) { return lens[x] > lens[y]; });
+        int32_t off = 0, slot = 0;
+        for (int i = 0; i < batch; ++i) {
+            const int32_t b = pa.row[i];
+            const int32_t nch = row_chunks((lens[b] + kPageSize - 1) / kPageSize, (int)T);
+            pa.len[i] = lens[b];
+            pa.off[i] = off;
+            pa.nch[i] = nch;
+            pa.slot[i] = slot;
+            off += nch;
+            if (nch > 1) slot += nch;
         }
     }
     noalloc_plan_kernel<<<1, 1024, 0, st>>>(pa);

@@ -184,7 +184,7 @@ def test_footprint_query_equals_eq1_when_lengths_fill_pages(kvlib):
 def test_split_pages_range(kvlib):
     h = host_cache(kvlib)
     kvlib.kv_cache_set_split_pages(h, 0)
-    kvlib.kv_cache_set_split_pages(h, 64)
+    kvlib.kv_cache_set_split_pages(h, 1024)
     with pytest.raises(kvlib.KVDecodeError):
-        kvlib.kv_cache_set_split_pages(h, 65)
+        kvlib.kv_cache_set_split_pages(h, 1025)
     kvlib.kv_cache_destroy(h)

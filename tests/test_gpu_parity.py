@@ -91,10 +91,13 @@ SMALL = [
     ("gqa7_64", 14, 2, 64, [3, 16, 33, 250]),
     ("gqa8_64", 8, 1, 64, [5, 64, 129]),
     ("gqa2_128", 4, 2, 128, [17, 100, 1000]),
+    # rows longer than a 32-page id window, and longer than 32 items at small splits
+    ("mha64_long", 8, 8, 64, [3000, 40]),
+    ("gqa7_long", 28, 4, 128, [4000, 5]),
 ]
 
 
-@pytest.mark.parametrize("split", [0, 1, 3, 64])
+@pytest.mark.parametrize("split", [0, 1, 3, 64, 1024])
 @pytest.mark.parametrize("name,Hq,Hkv,d,lens", SMALL)
 def test_decode_matches_oracle_small(name, Hq, Hkv, d, lens, split):
     cfg = wl.custom(name, 2, Hq, Hkv, d, len(lens), lens=lens, seed=31 + Hq + d, page_order="shuffled")
