@@ -208,14 +208,26 @@ def run_gpu(args, rank, world):
         f"{sess.query().pool_bytes / 2**30:.1f} GiB")
 
     def step(events=None):
+        """One decode step.  events: per-step event list to time the attention
+        launches.  Unfused: a pair around every decode_attention.  Fused: one
+        event after kv_begin_step and one after the last layer (the fused
+        launches are PDL-chained, and an event between two of them would cut
+        the overlap), so a launch's time is the span over L."""
         sess.begin_step()
+        if events is not None and not args.unfused:
+            events[0].record(stream)
         for l in range(L):
-            sess.append(l, ks[l], vs[l])
-            if events is not None:
-                events[l][0].record(stream)
-            sess.attend(l, qs[l], outs[l])
-            if events is not None:
-                events[l][1].record(stream)
+            if args.unfused:
+                sess.append(l, ks[l], vs[l])
+                if events is not None:
+                    events[2 * l].record(stream)
+                sess.attend(l, qs[l], outs[l])
+                if events is not None:
+                    events[2 * l + 1].record(stream)
+            else:
+                sess.append_attend(l, qs[l], ks[l], vs[l], outs[l])
+        if events is not None and not args.unfused:
+            events[1].record(stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -224,8 +236,8 @@ def run_gpu(args, rank, world):
 
     # ---- device-timed region
     attended_per_step = []
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(L)]
-          for _ in range(args.steps)]
+    n_ev = 2 * L if args.unfused else 2
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
@@ -242,13 +254,16 @@ def run_gpu(args, rank, world):
     if world > 1:
         torch.distributed.barrier()
     ms = start.elapsed_time(stop)
-    attn_ms = [e0.elapsed_time(e1) for evs in ev for (e0, e1) in evs]
+    if args.unfused:
+        attn_ms = [evs[2 * l].elapsed_time(evs[2 * l + 1]) for evs in ev for l in range(L)]
+    else:
+        attn_ms = [evs[0].elapsed_time(evs[1]) / L for evs in ev]
     step_bytes = []
     attn_bytes = []
     for att in attended_per_step:
         a, p = layer_bytes(cfg, att)
         step_bytes.append(L * (a + p))
-        attn_bytes.append(a)
+        attn_bytes.append(a if args.unfused else a + p)   # the fused kernel also writes the new K/V
     st = sess.query()
     assert st.device_error == 0, st.device_error
 
@@ -283,8 +298,11 @@ def run_gpu(args, rank, world):
                     dv[l].copy_(hv[l], non_blocking=True)
                 sess.begin_step()
                 for l in range(L):
-                    sess.append(l, dk[l], dv[l])
-                    sess.attend(l, dq[l], outs[l])
+                    if args.unfused:
+                        sess.append(l, dk[l], dv[l])
+                        sess.attend(l, dq[l], outs[l])
+                    else:
+                        sess.append_attend(l, dq[l], dk[l], dv[l], outs[l])
                     ho[l].copy_(outs[l], non_blocking=True)
             s1.record(stream)
         stream.synchronize()
@@ -316,6 +334,8 @@ def main():
     ap.add_argument("--config", default="llava", choices=["tiny", "llava", "qwen", "ragged", "long"])
     ap.add_argument("--phys-layers", type=int, default=0, help="layer pools held (profiling on a smaller cache)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--unfused", action="store_true",
+                    help="kv_append and decode_attention as two launches per layer (default: one fused launch)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     args = ap.parse_args()
@@ -383,12 +403,15 @@ def main():
         "steps_per_s": round(steps_per_s * 1.0, 3),
         "pct_of_measured_hbm": round(100 * gbs / world / peak, 2),
         "pct_of_nominal_8tbs": round(100 * gbs / world / NOMINAL_HBM_GBS, 2),
-        "roofline": {"bound": "hbm", "kernel": "decode_attention", "achieved": round(achieved, 2),
+        "roofline": {"bound": "hbm", "kernel": "decode_attention" if args.unfused else "decode_attention_append",
+                     "achieved": round(achieved, 2),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "traffic": (traffic["dram_bytes_per_launch_full"] if traffic else None),
                      "algorithmic_bytes_per_launch": int(attn_bytes), "avg_launch_ms": round(attn_ms, 4)},
         "clocks": r["clocks"],
-        "gpu_launches": args.steps * (1 + 2 * L),
+        "gpu_launches": args.steps * (1 + (2 if args.unfused else 1) * L),
+        "step_kernels": "kv_begin_step + per layer " + ("kv_append, decode_attention" if args.unfused
+                                                          else "decode_attention_append (fused, PDL)"),
     }
     if r["e2e"]:
         e = r["e2e"]

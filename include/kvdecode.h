@@ -192,6 +192,22 @@ KVC_API int kv_append(kv_cache *cache, int32_t layer, int32_t batch, const void 
 KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, const void *q, void *out,
                      float softmax_scale, void *stream);
 
+/* kv_append and decode_attention of one layer in a single kernel: the new
+ * token's K and V (k_new, v_new: device [batch][H_kv][d_h] bf16) are written
+ * into position s_b of each sequence and used in place of that slot's old
+ * contents while the layer's pages stream through shared memory.  Same
+ * result and cache contents as kv_append followed by decode_attention.
+ * The kernel is launched with programmatic dependent launch: it may start,
+ * and stream this layer's cached pages (positions < s_b), while the kernel
+ * launched just before it on `stream` is finishing; it reads q, k_new and
+ * v_new and writes anything only after that kernel has completed.  So the
+ * kernel launched just before it must not write this layer's cached pages
+ * (none of this library's kernels does; a foreign kernel could only do so if
+ * it signalled its dependents early). */
+KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batch, const void *q,
+                                    const void *k_new, const void *v_new, void *out,
+                                    float softmax_scale, void *stream);
+
 /* ------------------------------------------------ allocation-free decode -- */
 
 /* decode_attention for callers that may not allocate device memory while they

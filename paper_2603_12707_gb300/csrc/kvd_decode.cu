@@ -457,7 +457,27 @@ struct GqaCompute {
     }
 };
 
-template <int D, bool GQA>
+// The new token of row (en.b, g) into row r of the staged K and V tiles and
+// into the pool (fused append): lanes 0..CH-1 move K, CH..2CH-1 move V.
+template <int D>
+__device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanEntry& en, int g, int32_t pid,
+                                              uint8_t* sK, uint8_t* sV, int lane)
+{
+    constexpr int CH = D / 8;
+    const int r = (en.len - 1) % kPageSize;
+    if (lane < 2 * CH) {
+        const bool is_k = lane < CH;
+        const int c = is_k ? lane : lane - CH;
+        const int64_t src = ((int64_t)en.b * p.H_kv + g) * D + c * 8;
+        const uint4 v = *reinterpret_cast<const uint4*>((is_k ? p.k_new : p.v_new) + src);
+        *reinterpret_cast<uint4*>((is_k ? sK : sV) + swz(r, c)) = v;
+        const int64_t dst = (((int64_t)pid * p.H_kv + g) * kPageSize + r) * D + c * 8;
+        *reinterpret_cast<uint4*>((is_k ? p.pool_k : p.pool_v) + dst) = v;
+    }
+    __syncwarp();
+}
+
+template <int D, bool GQA, bool FUSED>
 __global__ void __launch_bounds__(kWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                   const DecodeParams p)
@@ -494,6 +514,10 @@ __global__ void __launch_bounds__(kWarps * 32)
 
     using Comp = typename std::conditional<GQA, GqaCompute<D>, MhaCompute<D>>::type;
     Comp comp;
+    // Fused launches depend programmatically on the previous kernel: until
+    // griddep_wait() only the plan, page table and cache pages (none of which
+    // that kernel writes) are read; q, k_new, v_new and every write come after.
+    bool waited = !FUSED;
 
     int item = 0;
     if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
@@ -541,6 +565,11 @@ __global__ void __launch_bounds__(kWarps * 32)
         __syncwarp();
         for (int j = 0; j < pre; ++j) issue(j, j);
         pending = (1u << pre) - 1u;
+        if (!waited) {
+            griddep_wait();
+            griddep_launch_dependents();
+            waited = true;
+        }
         comp.start(p, en, g, lane);
 
         for (int j = 0; j < np; ++j) {
@@ -554,6 +583,11 @@ __global__ void __launch_bounds__(kWarps * 32)
             pending &= ~(1u << s);
             const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
             uint8_t* sK = ring + s * STAGE;
+            if constexpr (FUSED) {
+                // the issue side has not moved past this page's id window
+                if (en.chunk == en.n_chunks - 1 && j == np - 1)
+                    put_new_token<D>(p, en, g, __shfl_sync(0xffffffffu, pid_cur, j & 31), sK, sK + TILE, lane);
+            }
             comp.page(sK, sK + TILE, ring_s + s * STAGE, ring_s + s * STAGE + TILE, valid, p.scale_log2, lane);
             fence_proxy_async_smem();
             __syncwarp();
@@ -588,10 +622,10 @@ __global__ void __launch_bounds__(kWarps * 32)
     }
 }
 
-template <int D, bool GQA>
+template <int D, bool GQA, bool FUSED>
 cudaError_t prepare_variant()
 {
-    static cudaError_t status = cudaFuncSetAttribute(decode_kernel<D, GQA>,
+    static cudaError_t status = cudaFuncSetAttribute(decode_kernel<D, GQA, FUSED>,
                                                      cudaFuncAttributeMaxDynamicSharedMemorySize, Geo<D>::kSmem);
     return status;
 }
@@ -599,22 +633,38 @@ cudaError_t prepare_variant()
 template <int D, bool GQA>
 cudaError_t variant_info(DecodeVariant* v)
 {
-    cudaError_t e = prepare_variant<D, GQA>();
+    cudaError_t e = prepare_variant<D, GQA, false>();
+    if (e == cudaSuccess) e = prepare_variant<D, GQA, true>();
     if (e != cudaSuccess) return e;
     v->warps = kWarps;
     v->smem_bytes = Geo<D>::kSmem;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v->ctas_per_sm, decode_kernel<D, GQA>, kWarps * 32,
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v->ctas_per_sm, decode_kernel<D, GQA, false>, kWarps * 32,
                                                          Geo<D>::kSmem);
 }
 
 template <int D, bool GQA>
-cudaError_t launch_variant(int grid, const CUtensorMap& tk, const CUtensorMap& tv, const DecodeParams& p,
-                           cudaStream_t st)
+cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+                           const DecodeParams& p, cudaStream_t st)
 {
-    cudaError_t e = prepare_variant<D, GQA>();
+    if (!fused) {
+        cudaError_t e = prepare_variant<D, GQA, false>();
+        if (e != cudaSuccess) return e;
+        decode_kernel<D, GQA, false><<<grid, kWarps * 32, Geo<D>::kSmem, st>>>(tk, tv, p);
+        return cudaGetLastError();
+    }
+    cudaError_t e = prepare_variant<D, GQA, true>();
     if (e != cudaSuccess) return e;
-    decode_kernel<D, GQA><<<grid, kWarps * 32, Geo<D>::kSmem, st>>>(tk, tv, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kWarps * 32);
+    cfg.dynamicSmemBytes = Geo<D>::kSmem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, decode_kernel<D, GQA, true>, tk, tv, p);
 }
 
 }  // namespace
@@ -626,13 +676,13 @@ cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v)
     return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_decode(int D, bool gqa, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+cudaError_t launch_decode(int D, bool gqa, bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
                           const DecodeParams& p, cudaStream_t st)
 {
-    if (D == 128) return gqa ? launch_variant<128, true>(grid, tk, tv, p, st)
-                             : launch_variant<128, false>(grid, tk, tv, p, st);
-    if (D == 64) return gqa ? launch_variant<64, true>(grid, tk, tv, p, st)
-                            : launch_variant<64, false>(grid, tk, tv, p, st);
+    if (D == 128) return gqa ? launch_variant<128, true>(fused, grid, tk, tv, p, st)
+                             : launch_variant<128, false>(fused, grid, tk, tv, p, st);
+    if (D == 64) return gqa ? launch_variant<64, true>(fused, grid, tk, tv, p, st)
+                            : launch_variant<64, false>(fused, grid, tk, tv, p, st);
     return cudaErrorInvalidValue;
 }
 

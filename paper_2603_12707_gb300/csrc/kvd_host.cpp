@@ -77,7 +77,8 @@ struct kv_cache {
     int32_t* meta = nullptr;                    // page table [max_seqs][max_pages], then seq_len [max_seqs]
     int32_t* step_seq = nullptr;
     int32_t* tickets = nullptr;
-    uint32_t* queue = nullptr;
+    uint32_t* queue = nullptr;                  // two (next item, warps done) counter pairs
+    uint32_t fused_launches = 0;                // fused launches alternate counter pairs
     int32_t* err = nullptr;
     PlanEntry* plan = nullptr;
     int64_t plan_cap = 0;
@@ -252,14 +253,14 @@ int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
         KVD_CUDA_C(cudaMalloc((void**)&c->meta, meta_elems * sizeof(int32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->step_seq, (size_t)k.max_seqs * sizeof(int32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->tickets, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t)));
-        KVD_CUDA_C(cudaMalloc((void**)&c->queue, 2 * sizeof(uint32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->queue, 4 * sizeof(uint32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->err, sizeof(int32_t)));
         KVD_CUDA_C(cudaMemsetAsync(c->pools, 0, pool_bytes, st));
         KVD_CUDA_C(cudaMemsetAsync(c->meta, 0xff, (size_t)k.max_seqs * k.max_pages_per_seq * sizeof(int32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->seq_len_dev(), 0, (size_t)k.max_seqs * sizeof(int32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->step_seq, 0, (size_t)k.max_seqs * sizeof(int32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->tickets, 0, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t), st));
-        KVD_CUDA_C(cudaMemsetAsync(c->queue, 0, 2 * sizeof(uint32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->queue, 0, 4 * sizeof(uint32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->err, 0, sizeof(int32_t), st));
 #undef KVD_CUDA_C
 
@@ -585,14 +586,17 @@ int kv_append(kv_cache* c, int32_t layer, int32_t batch, const void* k_new, cons
     return KVC_OK;
 }
 
-int decode_attention(kv_cache* c, int32_t layer, int32_t batch, const void* q, void* out, float softmax_scale,
-                     void* stream)
+static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_t batch, const void* q,
+                            const void* k_new, const void* v_new, void* out, float softmax_scale, void* stream)
 {
-    if (int rc = check_step(c, "decode_attention", layer, batch)) return rc;
+    if (int rc = check_step(c, what, layer, batch)) return rc;
+    const bool fused = k_new != nullptr;
     if (!q || !out || !aligned16(q) || !aligned16(out))
-        return fail(KVC_ERR_INVALID, "decode_attention: q / out must be non-null and 16-byte aligned");
+        return fail(KVC_ERR_INVALID, std::string(what) + ": q / out must be non-null and 16-byte aligned");
+    if (fused && (!v_new || !aligned16(k_new) || !aligned16(v_new)))
+        return fail(KVC_ERR_INVALID, std::string(what) + ": k_new / v_new must be non-null and 16-byte aligned");
     if (!(softmax_scale <= 0.f) && !std::isfinite(softmax_scale))
-        return fail(KVC_ERR_INVALID, "decode_attention: softmax_scale must be finite");
+        return fail(KVC_ERR_INVALID, std::string(what) + ": softmax_scale must be finite");
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)c->cfg.head_dim);
     DecodeParams p;
     p.q = static_cast<const uint16_t*>(q);
@@ -602,7 +606,9 @@ int decode_attention(kv_cache* c, int32_t layer, int32_t batch, const void* q, v
     p.part_o = c->part_o;
     p.part_ml = c->part_ml;
     p.tickets = c->tickets;
-    p.queue = c->queue;
+    // A fused launch may start while the previous one drains, so consecutive
+    // fused launches use different work counters.
+    p.queue = c->queue + (fused ? 2 * (c->fused_launches & 1u) : 0);
     p.err = c->err;
     p.num_pages = c->cfg.num_pages;
     p.n_items = c->step_entries * c->cfg.num_kv_heads;
@@ -611,12 +617,30 @@ int decode_attention(kv_cache* c, int32_t layer, int32_t batch, const void* q, v
     p.G = c->group;
     p.max_pages = c->cfg.max_pages_per_seq;
     p.scale_log2 = scale * 1.4426950408889634f;
+    p.k_new = static_cast<const uint16_t*>(k_new);
+    p.v_new = static_cast<const uint16_t*>(v_new);
+    p.pool_k = c->k_pool(layer);
+    p.pool_v = c->v_pool(layer);
     const int64_t resident = (int64_t)c->num_sms * std::max(1, c->variant.ctas_per_sm);
     const int64_t want = (p.n_items + c->variant.warps - 1) / c->variant.warps;
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
-    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, grid, c->tmaps[2 * layer], c->tmaps[2 * layer + 1], p,
-                           static_cast<cudaStream_t>(stream)));
+    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[2 * layer], c->tmaps[2 * layer + 1],
+                           p, static_cast<cudaStream_t>(stream)));
+    if (fused) ++c->fused_launches;
     return KVC_OK;
+}
+
+int decode_attention(kv_cache* c, int32_t layer, int32_t batch, const void* q, void* out, float softmax_scale,
+                     void* stream)
+{
+    return launch_attention(c, "decode_attention", layer, batch, q, nullptr, nullptr, out, softmax_scale, stream);
+}
+
+int decode_attention_append(kv_cache* c, int32_t layer, int32_t batch, const void* q, const void* k_new,
+                            const void* v_new, void* out, float softmax_scale, void* stream)
+{
+    if (!k_new) return fail(KVC_ERR_INVALID, "decode_attention_append: k_new must be non-null");
+    return launch_attention(c, "decode_attention_append", layer, batch, q, k_new, v_new, out, softmax_scale, stream);
 }
 
 }  // extern "C"

@@ -116,6 +116,13 @@ struct DecodeParams {
     int32_t n_items;
     int32_t H_kv, H_q, G, max_pages;
     float scale_log2;         // softmax scale * log2(e)
+    // Fused append (decode_attention_append only): the step's new K/V rows,
+    // written into slot len-1 of each row's last page and used in place of
+    // what the page held there.
+    const uint16_t* k_new;    // [B][H_kv][D] bf16
+    const uint16_t* v_new;
+    uint16_t* pool_k;         // this layer's pools [num_pages][H_kv][P][D]
+    uint16_t* pool_v;
 };
 
 // Message returned by kv_last_error() on the calling thread.
@@ -134,7 +141,10 @@ struct DecodeVariant {
     int ctas_per_sm;  // occupancy at that shared memory
 };
 cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v);
-cudaError_t launch_decode(int D, bool gqa, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+// fused: the append + attention kernel, launched with programmatic dependent
+// launch (it streams its first pages before the previous kernel finishes and
+// reads q / k_new / v_new and writes anything only after it has).
+cudaError_t launch_decode(int D, bool gqa, bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
                           const DecodeParams& p, cudaStream_t st);
 
 }  // namespace kvd

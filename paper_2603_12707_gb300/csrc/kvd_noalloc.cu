@@ -252,10 +252,12 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.G = G;
     p.max_pages = max_pages;
     p.scale_log2 = scale * 1.4426950408889634f;
+    p.k_new = p.v_new = nullptr;
+    p.pool_k = p.pool_v = nullptr;
     const int64_t resident = (int64_t)num_sms * std::max(1, var.ctas_per_sm);
     const int64_t want = (p.n_items + var.warps - 1) / var.warps;
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
-    if (cudaError_t e = launch_decode(head_dim, G > 1, grid, maps[0], maps[1], p, st); e != cudaSuccess)
+    if (cudaError_t e = launch_decode(head_dim, G > 1, false, grid, maps[0], maps[1], p, st); e != cudaSuccess)
         return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     return KVC_OK;
 }

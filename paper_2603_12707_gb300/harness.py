@@ -68,6 +68,11 @@ class DecodeSession:
     def attend(self, layer: int, q, out, scale: float = 0.0):
         kd.decode_attention(self.h, self.phys(layer), self.cfg.batch, q, out, scale, self.stream)
 
+    def append_attend(self, layer: int, q, k_new, v_new, out, scale: float = 0.0):
+        """kv_append + decode_attention of one layer in one fused launch."""
+        kd.decode_attention_append(self.h, self.phys(layer), self.cfg.batch, q, k_new, v_new, out, scale,
+                                   self.stream)
+
     def query(self, raise_on_device_error=True):
         return kd.kv_cache_query(self.h, raise_on_device_error)
 

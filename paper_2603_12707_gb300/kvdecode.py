@@ -72,6 +72,7 @@ _SIGS = {
     "kv_begin_step": [_P, _I32, _P, _P],
     "kv_append": [_P, _I32, _I32, _P, _P, _P],
     "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
+    "decode_attention_append": [_P, _I32, _I32, _P, _P, _P, _P, ctypes.c_float, _P],
     "decode_attention_noalloc": [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _I32, _P, _P, _P,
                                  ctypes.c_float, _P, _P],
 }
@@ -203,6 +204,12 @@ def kv_append(h, layer: int, batch: int, k_new, v_new, stream=None):
 def decode_attention(h, layer: int, batch: int, q, out, softmax_scale: float = 0.0, stream=None):
     _check(load().decode_attention(h, layer, batch, _ptr(q), _ptr(out), float(softmax_scale), _stream(stream)),
            "decode_attention")
+
+
+def decode_attention_append(h, layer: int, batch: int, q, k_new, v_new, out, softmax_scale: float = 0.0,
+                            stream=None):
+    _check(load().decode_attention_append(h, layer, batch, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(out),
+                                          float(softmax_scale), _stream(stream)), "decode_attention_append")
 
 
 def decode_attention_noalloc(k_pool, v_pool, num_pages: int, num_q_heads: int, num_kv_heads: int,

@@ -37,9 +37,9 @@ class Tracked:
     """A DecodeSession plus host copies of each layer pool's logical content."""
 
     def __init__(self, cfg, extra_tokens=8, lens=None, split_pages=0, layers_filled=None, keep_host=True,
-                 keep_rows=None):
+                 keep_rows=None, stream=None):
         self.cfg = cfg
-        self.sess = DecodeSession(cfg, extra_tokens=extra_tokens, lens=lens, split_pages=split_pages)
+        self.sess = DecodeSession(cfg, extra_tokens=extra_tokens, lens=lens, split_pages=split_pages, stream=stream)
         self.keep_host = keep_host
         self.keep_rows = list(range(cfg.batch)) if keep_rows is None else list(keep_rows)
         self.layers_filled = list(range(cfg.phys_layers)) if layers_filled is None else list(layers_filled)
@@ -59,13 +59,17 @@ class Tracked:
         self.sess.begin_step()
         self.step += 1
 
-    def run_layer(self, layer, scale=0.0):
-        """Append + attend one logical layer; returns (out bf16 tensor, q, k_new, v_new)."""
+    def run_layer(self, layer, scale=0.0, fused=False):
+        """Append + attend one logical layer (two launches, or the fused one);
+        returns (out bf16 tensor, q, k_new, v_new)."""
         cfg = self.cfg
         q, kn, vn = wl.step_inputs(cfg, self.step, layer, "cuda")
         out = torch.empty_like(q)
-        self.sess.append(layer, kn, vn)
-        self.sess.attend(layer, q, out, scale)
+        if fused:
+            self.sess.append_attend(layer, q, kn, vn, out, scale)
+        else:
+            self.sess.append(layer, kn, vn)
+            self.sess.attend(layer, q, out, scale)
         if self.keep_host:
             p = self.sess.phys(layer)
             kh, vh = u16(kn), u16(vn)

@@ -184,6 +184,63 @@ def test_step_and_attention_errors_do_not_launch():
     t.close()
 
 
+# ------------------------------------------------------ fused append + attend
+@pytest.mark.parametrize("name,Hq,Hkv,d,lens", [
+    ("mha128", 8, 8, 128, [0, 15, 16, 31, 200, 700]),
+    ("gqa7_128", 28, 4, 128, [0, 1, 16, 47, 300, 2100]),
+    ("mha64", 8, 8, 64, [3, 16, 129]),
+    ("gqa7_64", 14, 2, 64, [15, 33, 250]),
+])
+@pytest.mark.parametrize("split", [0, 1, 1024])
+def test_fused_append_attend_equals_append_then_attend(name, Hq, Hkv, d, lens, split):
+    """decode_attention_append: bit-identical output and cache contents to
+    kv_append + decode_attention, and the oracle's result, over several
+    steps (pages filling up and new pages taken)."""
+    outs = {}
+    pools = {}
+    for fused in (False, True):
+        cfg = wl.custom(name, 3, Hq, Hkv, d, len(lens), lens=lens, seed=41 + d, page_order="shuffled")
+        t = Tracked(cfg, extra_tokens=24, split_pages=split, keep_host=fused)
+        res = []
+        for step in range(4):
+            t.begin_step()
+            for layer in range(cfg.num_layers):
+                out, q, _, _ = t.run_layer(layer, fused=fused)
+                res.append(out.clone())
+                if fused and step in (0, 3):
+                    torch.cuda.synchronize()
+                    ref, vmax = t.oracle(layer, q)
+                    assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv, what=(name, split, step, layer))
+        torch.cuda.synchronize()
+        outs[fused] = res
+        pools[fused] = [device_pool(t.sess, l) for l in range(cfg.phys_layers)]
+        t.close()
+    for a, b in zip(outs[False], outs[True]):
+        assert torch.equal(a, b)
+    for (ka, va), (kb, vb) in zip(pools[False], pools[True]):
+        assert np.array_equal(ka, kb) and np.array_equal(va, vb)
+
+
+def test_fused_layers_back_to_back_on_one_stream():
+    """Consecutive fused launches overlap (each may start while the previous
+    drains): a whole multi-layer step on one side stream matches the oracle."""
+    cfg = wl.custom("pdl", 6, 28, 4, 128, 6, lens=[900, 33, 2500, 16, 400, 1200], seed=99, page_order="shuffled")
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        t = Tracked(cfg, extra_tokens=8, stream=stream)
+        for step in range(2):
+            t.begin_step()
+            got = []
+            for layer in range(cfg.num_layers):
+                out, q, _, _ = t.run_layer(layer, fused=True)
+                got.append((layer, out, q))
+            stream.synchronize()
+            for layer, out, q in got:
+                ref, vmax = t.oracle(layer, q)
+                assert_close(bf16_to_f64(out), ref, vmax, gqa=True, what=(step, layer))
+        t.close()
+
+
 # ------------------------------------------------------- decode: full size
 FULL = [
     # config, logical layers checked, sampled batch rows
@@ -201,8 +258,8 @@ def test_decode_matches_oracle_full_size(name, layers, rows):
     phys = sorted({l % cfg.phys_layers for l in layers})
     t = Tracked(cfg, extra_tokens=4, layers_filled=phys, keep_rows=rows)
     t.begin_step()
-    for layer in layers:
-        out, q, _, _ = t.run_layer(layer)
+    for i, layer in enumerate(layers):
+        out, q, _, _ = t.run_layer(layer, fused=(i % 2 == 1))
         torch.cuda.synchronize()
         r = list(range(cfg.batch)) if rows is None else rows
         ref, vmax = t.oracle(layer, q, rows=r)
