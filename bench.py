@@ -195,7 +195,8 @@ def run_gpu(args, rank, world):
     total_steps = args.warmup + args.steps + (args.steps if not args.no_e2e else 0) + 1
     t_setup = time.perf_counter()
     with torch.cuda.stream(stream):
-        sess = DecodeSession(cfg, extra_tokens=total_steps + 1, device="cuda", stream=stream)
+        sess = DecodeSession(cfg, extra_tokens=total_steps + 1, device="cuda", stream=stream,
+                             split_pages=args.split_pages)
         sess.fill_prefix()
         L, B = cfg.num_layers, cfg.batch
         qs, ks, vs = [], [], []
@@ -334,6 +335,8 @@ def main():
     ap.add_argument("--config", default="llava", choices=["tiny", "llava", "qwen", "ragged", "long"])
     ap.add_argument("--phys-layers", type=int, default=0, help="layer pools held (profiling on a smaller cache)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--split-pages", type=int, default=0,
+                    help="target pages per work item (0: the library's automatic choice)")
     ap.add_argument("--unfused", action="store_true",
                     help="kv_append and decode_attention as two launches per layer (default: one fused launch)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -399,6 +402,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {**describe(cfg), "l2": "each step streams the whole cache (far larger than the 129 MB L2)",
+                   "split_pages": args.split_pages or "auto",
                    "parallelism": f"replicas x{world}"},
         "steps_per_s": round(steps_per_s * 1.0, 3),
         "pct_of_measured_hbm": round(100 * gbs / world / peak, 2),

@@ -81,6 +81,7 @@ __global__ void __launch_bounds__(1024)
             chunk_range(np, nch, c, &first, &n);
             a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
         }
+        if (i < a.batch) a.rows[b] = make_int2(off, nch);
         carry += total;
     }
 }

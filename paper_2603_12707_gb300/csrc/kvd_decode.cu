@@ -9,9 +9,9 @@
 //   * the warp computes an online softmax over the item's tokens for the G
 //     query heads of the KV head (running max m in log2 units, running sum l,
 //     unnormalised accumulator o, all fp32);
-//   * a row with one item writes bf16 output directly; otherwise the item
-//     stores (o, m, l) as a partial and takes a ticket, and the warp that takes
-//     the row's last ticket merges the partials by log-sum-exp:
+//   * a row with one item writes bf16 output directly; otherwise each item
+//     stores (o, m, l) as a partial and a second pass (merge_kernel, one warp
+//     per (row, query head), one lane per item) merges them by log-sum-exp:
 //         M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c.
 // MHA (G = 1, 1 flop per byte) runs on the CUDA cores; GQA (2 <= G <= 8) runs
 // Q.K^T and P.V as m16n8k16 bf16 MMAs with the 16 tokens of a page as M and the
@@ -22,6 +22,7 @@
 // leaves.  Page ids outside the pool are recorded and replaced by page 0.
 #include <math.h>
 
+#include <algorithm>
 #include <type_traits>
 
 #include "kvd_internal.h"
@@ -32,8 +33,7 @@ namespace kvd {
 namespace {
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
-constexpr int kWarps = 4;
-constexpr int kMergeBytes = kMaxChunks * kMaxGroup * 8;   // per-warp (m, l) / weight table
+constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
 template <int D>
 struct Geo {
@@ -42,7 +42,7 @@ struct Geo {
     static constexpr int kStageBytes = 2 * kTileBytes;   // K tile + V tile
     static constexpr int kRing = (D == 128) ? 3 : 6;     // stages per warp
     static constexpr int kRingBytes = kWarps * kRing * kStageBytes;
-    static constexpr int kSmem = kRingBytes + kWarps * kMergeBytes + kWarps * kRing * 8 + 1024;
+    static constexpr int kSmem = kRingBytes + kWarps * kRing * 8 + 1024;
 };
 
 // Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r, for a tile that
@@ -75,126 +75,6 @@ __device__ __forceinline__ void axpy8(float (&o)[8], float p, const uint4& v)
     o[5] = fmaf(p, bf16hi(v.z), o[5]);
     o[6] = fmaf(p, bf16lo(v.w), o[6]);
     o[7] = fmaf(p, bf16hi(v.w), o[7]);
-}
-
-// Merge the partials of (row b, KV head g) into the bf16 output rows of its
-// G query heads.  One warp; `wsm` (kMergeBytes of the warp's shared memory)
-// holds the per-(chunk, head) weights.
-//   M_h = max_c m_ch,  w_ch = 2^(m_ch - M_h) / sum_c 2^(m_ch - M_h) l_ch,
-//   O_h = sum_c w_ch o_ch.
-// Loads are issued several chunks at a time so the merge is not bound by
-// one L2 round trip per chunk.
-template <int D, bool GQA>
-__device__ void merge_partials(const DecodeParams& p, const PlanEntry& en, int g, int lane, float* wsm)
-{
-    constexpr int PER = D / 32;                 // dims per lane
-    constexpr int HMAX = GQA ? kMaxGroup : 1;
-    constexpr int U = GQA ? 2 : 8;              // chunks in flight per round
-    const int G = GQA ? p.G : 1;
-    const int nch = en.n_chunks;
-    auto slot_of = [&](int c) { return ((int64_t)(en.slot_base + c) * p.H_kv + g) * G; };
-
-    for (int i = lane; i < nch * G; i += 32) {
-        const int c = i / G, h = i - c * G;
-        const float2 ml = __ldcg(&p.part_ml[slot_of(c) + h]);
-        wsm[2 * i] = ml.x;
-        wsm[2 * i + 1] = ml.y;
-    }
-    __syncwarp();
-    {
-        // lanes 4h .. 4h+3 reduce head h over chunks c = lane%4, +4, ...
-        const int h = lane >> 2, q4 = lane & 3;
-        float M = -INFINITY, L = 0.f;
-        if (h < G)
-            for (int c = q4; c < nch; c += 4) M = fmaxf(M, wsm[2 * (c * G + h)]);
-        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 1));
-        M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, 2));
-        if (h < G)
-            for (int c = q4; c < nch; c += 4) L = fmaf(ex2(wsm[2 * (c * G + h)] - M), wsm[2 * (c * G + h) + 1], L);
-        L += __shfl_xor_sync(0xffffffffu, L, 1);
-        L += __shfl_xor_sync(0xffffffffu, L, 2);
-        __syncwarp();
-        const float invL = 1.f / L;
-        if (h < G)
-            for (int c = q4; c < nch; c += 4) wsm[2 * (c * G + h)] = ex2(wsm[2 * (c * G + h)] - M) * invL;
-        __syncwarp();
-    }
-    float acc[HMAX][PER];
-#pragma unroll
-    for (int h = 0; h < HMAX; ++h)
-#pragma unroll
-        for (int k = 0; k < PER; ++k) acc[h][k] = 0.f;
-    for (int c0 = 0; c0 < nch; c0 += U) {
-        float v[U][HMAX][PER];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int c = c0 + u;
-#pragma unroll
-            for (int h = 0; h < HMAX; ++h) {
-                if (c < nch && h < G) {
-                    const float* po = p.part_o + (slot_of(c) + h) * D + lane * PER;
-                    if constexpr (PER == 4) {
-                        const float4 t = __ldcg(reinterpret_cast<const float4*>(po));
-                        v[u][h][0] = t.x; v[u][h][1] = t.y; v[u][h][2] = t.z; v[u][h][3] = t.w;
-                    } else {
-                        const float2 t = __ldcg(reinterpret_cast<const float2*>(po));
-                        v[u][h][0] = t.x; v[u][h][1] = t.y;
-                    }
-                } else {
-#pragma unroll
-                    for (int k = 0; k < PER; ++k) v[u][h][k] = 0.f;
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int c = c0 + u;
-#pragma unroll
-            for (int h = 0; h < HMAX; ++h) {
-                const float w = (c < nch && h < G) ? wsm[2 * (c * G + h)] : 0.f;
-#pragma unroll
-                for (int k = 0; k < PER; ++k) acc[h][k] = fmaf(w, v[u][h][k], acc[h][k]);
-            }
-        }
-    }
-#pragma unroll
-    for (int h = 0; h < HMAX; ++h) {
-        if (h < G) {
-            uint16_t* orow = p.out + ((int64_t)en.b * p.H_q + g * G + h) * D + lane * PER;
-            if constexpr (PER == 4) {
-                uint2 o;
-                o.x = pack_bf16(acc[h][0], acc[h][1]);
-                o.y = pack_bf16(acc[h][2], acc[h][3]);
-                *reinterpret_cast<uint2*>(orow) = o;
-            } else {
-                *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[h][0], acc[h][1]);
-            }
-        }
-    }
-    __syncwarp();
-}
-
-// Take the ticket of a finished split item whose partial the lanes have
-// stored; the warp that takes the row's last ticket merges.  One lane orders
-// the warp's stores before its ticket (the warp barrier makes the other
-// lanes' stores visible to it first); lane 31 is used because lane 0 issues
-// the TMA loads, which a fence in that lane might wait for.
-template <int D, bool GQA>
-__device__ __forceinline__ void take_ticket(const DecodeParams& p, const PlanEntry& en, int g, int lane, float* wsm)
-{
-    __syncwarp();
-    int last = 0;
-    int32_t* ticket = p.tickets + (int64_t)en.b * p.H_kv + g;
-    if (lane == 31) {
-        __threadfence();
-        last = (atomicAdd(ticket, 1) == en.n_chunks - 1);
-    }
-    last = __shfl_sync(0xffffffffu, last, 31);
-    if (last) {
-        __threadfence();
-        merge_partials<D, GQA>(p, en, g, lane, wsm);
-        if (lane == 31) *ticket = 0;   // ready for the next layer
-    }
 }
 
 // ------------------------------------------------------------ MHA, CUDA cores
@@ -271,9 +151,9 @@ struct MhaCompute {
         }
     }
 
-    // Writes the output (one item) or the partial (split row); returns true
-    // when a partial was stored and the row's ticket is due.
-    __device__ __forceinline__ bool finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    // Writes the output (a row of one item) or the item's partial (a split
+    // row; the merge pass combines them).
+    __device__ __forceinline__ void finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
     {
 #pragma unroll
         for (int mask = CH; mask < 32; mask <<= 1)
@@ -299,9 +179,7 @@ struct MhaCompute {
                 dst[1] = make_float4(o[4], o[5], o[6], o[7]);
             }
             if (lane == 0) p.part_ml[slot] = make_float2(m, l);
-            return true;
         }
-        return false;
     }
 };
 
@@ -408,7 +286,7 @@ struct GqaCompute {
         }
     }
 
-    __device__ __forceinline__ bool finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+    __device__ __forceinline__ void finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
     {
 #pragma unroll
         for (int mask = 4; mask < 32; mask <<= 1) {
@@ -451,9 +329,7 @@ struct GqaCompute {
                 if (h0 < G) p.part_ml[slot * G + h0] = make_float2(m0, l0);
                 if (h1 < G) p.part_ml[slot * G + h1] = make_float2(m1, l1);
             }
-            return true;
         }
-        return false;
     }
 };
 
@@ -492,8 +368,7 @@ __global__ void __launch_bounds__(kWarps * 32)
                                                ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t* ring = smem + warp * R * STAGE;
-    float* wsm = reinterpret_cast<float*>(smem + Gm::kRingBytes + warp * kMergeBytes);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Gm::kRingBytes + kWarps * kMergeBytes) + warp * R;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Gm::kRingBytes) + warp * R;
     const uint32_t ring_s = smem_addr(ring);
 
     if (lane == 0) {
@@ -597,9 +472,7 @@ __global__ void __launch_bounds__(kWarps * 32)
             }
         }
         if (!ok) break;
-        // Taking the ticket right away measured faster than deferring it
-        // behind the next item's first loads.
-        if (comp.finish(p, en, g, lane)) take_ticket<D, GQA>(p, en, g, lane, wsm);
+        comp.finish(p, en, g, lane);
         if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
         item = __shfl_sync(0xffffffffu, item, 0);
     }
@@ -618,6 +491,81 @@ __global__ void __launch_bounds__(kWarps * 32)
         if (atomicAdd(&p.queue[1], 1u) == total - 1) {
             p.queue[0] = 0;
             p.queue[1] = 0;
+        }
+    }
+}
+
+// Second pass.  Warp w handles (row b, query head h) = (w / H_q, w % H_q) of
+// a split row: lane c < n_chunks holds item c's (m, l); the weights
+// 2^(m_c - M) / sum_c 2^(m_c - M) l_c stay in registers and are broadcast
+// while the lanes (D/32 dims each) accumulate the items' o, eight items in
+// flight at a time.
+constexpr int kMergeWarps = 4;
+
+template <int D>
+__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodeParams p, int pdl)
+{
+    if (pdl) {
+        griddep_launch_dependents();   // the next layer may start streaming now
+        griddep_wait();                // the split pass of this layer is complete
+    }
+    constexpr int PER = D / 32;
+    const int lane = threadIdx.x & 31;
+    const int total = p.batch * p.H_q;
+    for (int w = blockIdx.x * kMergeWarps + (threadIdx.x >> 5); w < total; w += gridDim.x * kMergeWarps) {
+        const int b = w / p.H_q, h = w - b * p.H_q;
+        const int2 row = p.rows[b];
+        const int nch = row.y;
+        if (nch <= 1) continue;
+        const int g = h / p.G, hh = h - g * p.G;
+        auto slot = [&](int c) { return ((int64_t)(row.x + c) * p.H_kv + g) * p.G + hh; };
+        float m = -INFINITY, l = 0.f;
+        if (lane < nch) {
+            const float2 ml = __ldcg(&p.part_ml[slot(lane)]);
+            m = ml.x;
+            l = ml.y;
+        }
+        float M = m;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+        const float e = (lane < nch) ? ex2(m - M) : 0.f;
+        float L = e * l;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+        const float wgt = e / L;
+        float acc[PER];
+#pragma unroll
+        for (int k = 0; k < PER; ++k) acc[k] = 0.f;
+        for (int c0 = 0; c0 < nch; c0 += 8) {
+            float v[8][PER];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int c = c0 + u;
+                const float* po = p.part_o + slot(c < nch ? c : 0) * D + lane * PER;
+                if constexpr (PER == 4) {
+                    const float4 t = __ldcg(reinterpret_cast<const float4*>(po));
+                    v[u][0] = t.x; v[u][1] = t.y; v[u][2] = t.z; v[u][3] = t.w;
+                } else {
+                    const float2 t = __ldcg(reinterpret_cast<const float2*>(po));
+                    v[u][0] = t.x; v[u][1] = t.y;
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
+                if (c0 + u < nch)
+#pragma unroll
+                    for (int k = 0; k < PER; ++k) acc[k] = fmaf(wc, v[u][k], acc[k]);
+            }
+        }
+        uint16_t* orow = p.out + ((int64_t)b * p.H_q + h) * D + lane * PER;
+        if constexpr (PER == 4) {
+            uint2 o;
+            o.x = pack_bf16(acc[0], acc[1]);
+            o.y = pack_bf16(acc[2], acc[3]);
+            *reinterpret_cast<uint2*>(orow) = o;
+        } else {
+            *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0], acc[1]);
         }
     }
 }
@@ -668,6 +616,27 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
 }
 
 }  // namespace
+
+cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st)
+{
+    const int64_t warps = (int64_t)p.batch * p.H_q;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
+                                                                   (int64_t)num_sms * 16));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kMergeWarps * 32);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    const int flag = pdl ? 1 : 0;
+    if (D == 128) return cudaLaunchKernelEx(&cfg, merge_kernel<128>, p, flag);
+    if (D == 64) return cudaLaunchKernelEx(&cfg, merge_kernel<64>, p, flag);
+    return cudaErrorInvalidValue;
+}
 
 cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v)
 {

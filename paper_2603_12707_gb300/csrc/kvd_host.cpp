@@ -76,7 +76,7 @@ struct kv_cache {
     size_t layer_elems = 0;
     int32_t* meta = nullptr;                    // page table [max_seqs][max_pages], then seq_len [max_seqs]
     int32_t* step_seq = nullptr;
-    int32_t* tickets = nullptr;
+    int2* rows = nullptr;                       // per batch row: (first partial slot, items)
     uint32_t* queue = nullptr;                  // two (next item, warps done) counter pairs
     uint32_t fused_launches = 0;                // fused launches alternate counter pairs
     int32_t* err = nullptr;
@@ -89,6 +89,7 @@ struct kv_cache {
 
     // current step
     bool step_active = false;
+    bool step_split = false;                    // some row of the step has several items
     int32_t step_batch = 0;
     int32_t step_entries = 0;
     int32_t split_override = 0;
@@ -180,7 +181,7 @@ void release_device(kv_cache* c)
     cudaFree(c->pools);
     cudaFree(c->meta);
     cudaFree(c->step_seq);
-    cudaFree(c->tickets);
+    cudaFree(c->rows);
     cudaFree(c->queue);
     cudaFree(c->err);
     cudaFree(c->plan);
@@ -252,14 +253,14 @@ int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
         KVD_CUDA_C(cudaMalloc((void**)&c->pools, pool_bytes));
         KVD_CUDA_C(cudaMalloc((void**)&c->meta, meta_elems * sizeof(int32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->step_seq, (size_t)k.max_seqs * sizeof(int32_t)));
-        KVD_CUDA_C(cudaMalloc((void**)&c->tickets, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->rows, (size_t)k.max_seqs * sizeof(int2)));
         KVD_CUDA_C(cudaMalloc((void**)&c->queue, 4 * sizeof(uint32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->err, sizeof(int32_t)));
         KVD_CUDA_C(cudaMemsetAsync(c->pools, 0, pool_bytes, st));
         KVD_CUDA_C(cudaMemsetAsync(c->meta, 0xff, (size_t)k.max_seqs * k.max_pages_per_seq * sizeof(int32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->seq_len_dev(), 0, (size_t)k.max_seqs * sizeof(int32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->step_seq, 0, (size_t)k.max_seqs * sizeof(int32_t), st));
-        KVD_CUDA_C(cudaMemsetAsync(c->tickets, 0, (size_t)k.max_seqs * k.num_kv_heads * sizeof(int32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->rows, 0, (size_t)k.max_seqs * sizeof(int2), st));
         KVD_CUDA_C(cudaMemsetAsync(c->queue, 0, 4 * sizeof(uint32_t), st));
         KVD_CUDA_C(cudaMemsetAsync(c->err, 0, sizeof(int32_t), st));
 #undef KVD_CUDA_C
@@ -499,7 +500,12 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     }
     const int32_t T = c->split_override ? c->split_override : auto_item_pages(c, total_units);
     int64_t entries = 0;
-    for (int32_t b = 0; b < batch; ++b) entries += row_chunks(np_after[b], T);
+    bool split = false;
+    for (int32_t b = 0; b < batch; ++b) {
+        const int nch = row_chunks(np_after[b], T);
+        entries += nch;
+        split = split || nch > 1;
+    }
     if (!c->host_only)
         if (int rc = grow_scratch(c, entries, entries * c->cfg.num_kv_heads, static_cast<cudaStream_t>(stream)))
             return rc;
@@ -526,6 +532,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         pa.seq_len = c->seq_len_dev();
         pa.page_table = c->page_table();
         pa.plan = c->plan;
+        pa.rows = c->rows;
         pa.err = c->err;
         // Longest rows first: their items start early and the tail is short.
         pa.use_order = batch <= kPatchMax ? 1 : 0;
@@ -548,6 +555,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         }
     }
     c->step_active = true;
+    c->step_split = split;
     c->step_batch = batch;
     c->step_entries = (int32_t)entries;
     return KVC_OK;
@@ -605,7 +613,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.plan = c->plan;
     p.part_o = c->part_o;
     p.part_ml = c->part_ml;
-    p.tickets = c->tickets;
+    p.rows = c->rows;
+    p.batch = batch;
     // A fused launch may start while the previous one drains, so consecutive
     // fused launches use different work counters.
     p.queue = c->queue + (fused ? 2 * (c->fused_launches & 1u) : 0);
@@ -626,6 +635,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
     KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[2 * layer], c->tmaps[2 * layer + 1],
                            p, static_cast<cudaStream_t>(stream)));
+    if (c->step_split)
+        KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->num_sms, p, static_cast<cudaStream_t>(stream)));
     if (fused) ++c->fused_launches;
     return KVC_OK;
 }

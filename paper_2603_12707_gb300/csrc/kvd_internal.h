@@ -67,6 +67,7 @@ struct PlanArgs {
     int32_t* seq_len;    // [max_seqs]
     int32_t* page_table; // [max_seqs][max_pages]
     PlanEntry* plan;     // [n_entries]
+    int2* rows;          // [batch]: (first partial slot, items) of each batch row
     int32_t* err;
 };
 
@@ -109,7 +110,8 @@ struct DecodeParams {
     const PlanEntry* plan;
     float* part_o;            // [slots][G][D]
     float2* part_ml;          // [slots][G]  (running max in log2 units, sum)
-    int32_t* tickets;         // [batch][H_kv]
+    const int2* rows;         // [batch]: (first partial slot, items) per batch row
+    int32_t batch;
     uint32_t* queue;          // [0] next item, [1] warps finished
     int32_t* err;
     int64_t num_pages;
@@ -141,6 +143,10 @@ struct DecodeVariant {
     int ctas_per_sm;  // occupancy at that shared memory
 };
 cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v);
+// Second pass: log-sum-exp merge of the partials of every split row, one warp
+// per (row, query head).  pdl: launched with programmatic dependent launch
+// (it lets the next kernel start at once and waits for the split pass).
+cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st);
 // fused: the append + attention kernel, launched with programmatic dependent
 // launch (it streams its first pages before the previous kernel finishes and
 // reads q / k_new / v_new and writes anything only after it has).

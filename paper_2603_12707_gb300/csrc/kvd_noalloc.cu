@@ -10,8 +10,8 @@
 // not take the allocator's locks.  Those callers own the K/V pools and page
 // table themselves and call this entry point instead.
 //
-// Scratch.  The split plan, the per-item partial results, the merge tickets
-// and the work counters live in one file-scope __device__ array of
+// Scratch.  The split plan, the per-item partial results, the per-row merge
+// table and the work counters live in one file-scope __device__ array of
 // kNoAllocScratchBytes (16 MiB) that every GPU loading this library holds
 // until the process exits.  Host code cannot use the array's name as a device
 // address; the first call on each device looks the address up with
@@ -39,9 +39,8 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes]
 
 struct NoAllocPlanArgs {
     int32_t batch;
-    int32_t n_tickets;     // batch * H_kv
     PlanEntry* plan;
-    int32_t* tickets;
+    int2* rows;            // [batch]: (first partial slot, items)
     uint32_t* queue;
     int32_t* err;
     int32_t clear_err;
@@ -53,11 +52,10 @@ struct NoAllocPlanArgs {
     int32_t slot[kNoAllocMaxBatch];  // first partial slot (rows with one item use none)
 };
 
-// One block: clear the tickets and work counters, then write each row's
-// items (near-equal page ranges) at the offsets the host computed.
+// One block: clear the work counters, then write each row's items
+// (near-equal page ranges) at the offsets the host computed.
 __global__ void __launch_bounds__(1024) noalloc_plan_kernel(const __grid_constant__ NoAllocPlanArgs a)
 {
-    for (int i = threadIdx.x; i < a.n_tickets; i += blockDim.x) a.tickets[i] = 0;
     if (threadIdx.x == 0) {
         a.queue[0] = 0;
         a.queue[1] = 0;
@@ -70,6 +68,7 @@ __global__ void __launch_bounds__(1024) noalloc_plan_kernel(const __grid_constan
             chunk_range(np, a.nch[i], c, &first, &n);
             a.plan[a.off[i] + c] = PlanEntry{a.row[i], a.row[i], a.len[i], first, n, c, a.nch[i], a.slot[i]};
         }
+        a.rows[a.row[i]] = make_int2(a.slot[i], a.nch[i]);
     }
 }
 
@@ -172,7 +171,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     const int64_t warps = (int64_t)num_sms * std::max(1, var.ctas_per_sm) * std::max(1, var.warps);
     int64_t T = std::min<int64_t>(128, std::max<int64_t>(2, (total_pages * num_kv_heads + 3 * warps - 1) / (3 * warps)));
     int64_t entries = 0;
-    size_t off_o = 0, off_ml = 0, off_tk = 0, off_q = 0, off_err = 0, need = 0;
+    bool split_rows = false;
+    size_t off_o = 0, off_ml = 0, off_rows = 0, off_q = 0, off_err = 0, need = 0;
     for (;; T *= 2) {
         entries = 0;
         int64_t split_items = 0;   // only rows cut into several items keep partials
@@ -181,11 +181,12 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
             entries += nch;
             if (nch > 1) split_items += nch;
         }
+        split_rows = split_items > 0;
         const int64_t slots = split_items * num_kv_heads;
         off_o = round256((size_t)entries * sizeof(PlanEntry));
         off_ml = round256(off_o + (size_t)slots * G * head_dim * sizeof(float));
-        off_tk = round256(off_ml + (size_t)slots * G * sizeof(float2));
-        off_q = round256(off_tk + (size_t)batch * num_kv_heads * sizeof(int32_t));
+        off_rows = round256(off_ml + (size_t)slots * G * sizeof(float2));
+        off_q = round256(off_rows + (size_t)batch * sizeof(int2));
         off_err = off_q + 2 * sizeof(uint32_t);
         need = round256(off_err + sizeof(int32_t));
         if (need <= kNoAllocScratchBytes || T >= kMaxItemPages) break;
@@ -210,9 +211,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
 
     NoAllocPlanArgs pa;
     pa.batch = batch;
-    pa.n_tickets = batch * num_kv_heads;
     pa.plan = reinterpret_cast<PlanEntry*>(scratch);
-    pa.tickets = reinterpret_cast<int32_t*>(scratch + off_tk);
+    pa.rows = reinterpret_cast<int2*>(scratch + off_rows);
     pa.queue = reinterpret_cast<uint32_t*>(scratch + off_q);
     pa.err = device_error ? device_error : reinterpret_cast<int32_t*>(scratch + off_err);
     pa.clear_err = device_error ? 0 : 1;
@@ -242,7 +242,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.plan = pa.plan;
     p.part_o = reinterpret_cast<float*>(scratch + off_o);
     p.part_ml = reinterpret_cast<float2*>(scratch + off_ml);
-    p.tickets = pa.tickets;
+    p.rows = pa.rows;
+    p.batch = batch;
     p.queue = pa.queue;
     p.err = pa.err;
     p.num_pages = num_pages;
@@ -259,5 +260,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
     if (cudaError_t e = launch_decode(head_dim, G > 1, false, grid, maps[0], maps[1], p, st); e != cudaSuccess)
         return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
+    if (split_rows)
+        if (cudaError_t e = launch_merge(head_dim, false, num_sms, p, st); e != cudaSuccess)
+            return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     return KVC_OK;
 }
