@@ -1,5 +1,7 @@
 // Page-table maintenance, the per-step update and split plan, token writes /
 // reads into pages, and the fused K+V append (kv_append).
+#include <algorithm>
+
 #include "kvd_internal.h"
 
 namespace kvd {
@@ -146,7 +148,31 @@ __global__ void append_kernel(const AppendArgs a)
     *reinterpret_cast<uint4*>(a.pool_v + poff) = vv;
 }
 
+// One warp per plan entry: its page ids, contiguous, at entry * stride.
+__global__ void gather_pages_kernel(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
+                                    int32_t max_pages, int32_t* item_pages, int32_t stride)
+{
+    const int lane = threadIdx.x & 31;
+    const int warps = (gridDim.x * blockDim.x) >> 5;
+    for (int e = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; e < entries; e += warps) {
+        const PlanEntry en = plan[e];
+        const int32_t* src = page_table + (int64_t)en.seq * max_pages + en.first_page;
+        int32_t* dst = item_pages + (int64_t)e * stride;
+        for (int i = lane; i < en.n_pages; i += 32) dst[i] = src[i];
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
+                                int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st)
+{
+    if (entries <= 0) return cudaSuccess;
+    const int64_t want = ((int64_t)entries + 7) / 8;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * 8));
+    gather_pages_kernel<<<grid, 256, 0, st>>>(plan, entries, page_table, max_pages, item_pages, stride);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st)
 {

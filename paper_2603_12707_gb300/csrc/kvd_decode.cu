@@ -35,18 +35,19 @@ namespace {
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
-template <int D>
+template <int D, bool GQA>
 struct Geo {
-    static constexpr int kBoxes = D / 64;                // 64-column TMA boxes per tile
     static constexpr int kTileBytes = kPageSize * D * 2; // one (page, head) tile
     static constexpr int kStageBytes = 2 * kTileBytes;   // K tile + V tile
-    static constexpr int kRing = (D == 128) ? 3 : 6;     // stages per warp
+    // stages per warp (8 one-warp CTAs per SM); deeper rings with fewer warps
+    // measured slower for both paths
+    static constexpr int kRing = D == 128 ? 3 : 6;
     static constexpr int kRingBytes = kWarps * kRing * kStageBytes;
     static constexpr int kSmem = kRingBytes + kWarps * kRing * 8 + 1024;
 };
 
-// Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r, for a tile that
-// TMA wrote as [16 rows][64 cols] boxes (2 KiB each) with 128-byte swizzle.
+// Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r: TMA writes a
+// tile as D/64 blocks of [16 rows][64 cols] (2 KiB each), 128-byte swizzle.
 __device__ __forceinline__ uint32_t swz(int r, int c)
 {
     return (uint32_t)((c >> 3) * 2048 + r * 128 + (((c & 7) ^ (r & 7)) << 4));
@@ -358,7 +359,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                   const DecodeParams p)
 {
-    using Gm = Geo<D>;
+    using Gm = Geo<D, GQA>;
     constexpr int R = Gm::kRing;
     constexpr int STAGE = Gm::kStageBytes;
     constexpr int TILE = Gm::kTileBytes;
@@ -394,49 +395,47 @@ __global__ void __launch_bounds__(kWarps * 32)
     // that kernel writes) are read; q, k_new, v_new and every write come after.
     bool waited = !FUSED;
 
-    int item = 0;
-    if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
-    item = __shfl_sync(0xffffffffu, item, 0);
+    // The first item of every warp is its global warp index; later ones come
+    // from the work counter, offset by the number of warps.
+    const int n_warps = (int)gridDim.x * kWarps;
+    int item = (int)blockIdx.x * kWarps + warp;
 
     while (item < p.n_items) {
         const int e = item / p.H_kv;
         const int g = item - e * p.H_kv;
-        const PlanEntry en = p.plan[e];
-        const int np = en.n_pages;
-
-        // Page ids of the item in windows of 32: lane i holds page w*32 + i of
-        // the current window; the next window is fetched 24 pages ahead.
-        const int32_t* pt_row = p.page_table + (int64_t)en.seq * p.max_pages + en.first_page;
-        auto load_window = [&](int w0) {
-            int32_t v = (w0 + lane < np) ? pt_row[w0 + lane] : 0;
-            if (v < 0 || v >= p.num_pages) {
-                atomicOr(p.err, 1);
-                v = 0;
-            }
-            return v;
-        };
+        // The entry's page ids sit at a fixed stride, so they load alongside
+        // the entry.  Windows of 32: lane i holds page w*32 + i of the current
+        // window; the next window is fetched 24 pages ahead.
+        const int32_t* pt_row = p.item_pages + (int64_t)e * p.page_stride;
+        auto load_window = [&](int w0) { return (w0 + lane < p.page_stride) ? pt_row[w0 + lane] : 0; };
         int32_t pid_cur = load_window(0);
         int32_t pid_next = 0;
+        const PlanEntry en = p.plan[e];
+        const int np = en.n_pages;
 
         auto issue = [&](int j, int s) {
             if ((j & 31) == 8 && j + 24 < np) pid_next = load_window(j + 24);
             if ((j & 31) == 0 && j > 0) pid_cur = pid_next;
-            const int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
+            int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
+            if (pid < 0 || pid >= p.num_pages) {
+                if (lane == 0) atomicOr(p.err, 1);
+                pid = 0;
+            }
             if (lane == 0) {
                 const uint32_t bar = smem_addr(&bars[s]);
                 const uint32_t dst = ring_s + s * STAGE;
                 const int32_t y = (pid * p.H_kv + g) * kPageSize;
                 mbar_arrive_expect_tx(bar, STAGE);
-#pragma unroll
-                for (int bx = 0; bx < Gm::kBoxes; ++bx) {
-                    tma_load_2d(dst + bx * 2048, &tmk, bx * 64, y, bar, policy);
-                    tma_load_2d(dst + TILE + bx * 2048, &tmv, bx * 64, y, bar, policy);
+                if (p.kv_map) {
+                    tma_load_4d(dst, &tmk, 0, y, 0, 0, bar, policy);
+                } else {
+                    tma_load_3d(dst, &tmk, 0, y, 0, bar, policy);
+                    tma_load_3d(dst + TILE, &tmv, 0, y, 0, bar, policy);
                 }
             }
         };
 
         const int pre = np < R ? np : R;
-        fence_proxy_async_smem();
         __syncwarp();
         for (int j = 0; j < pre; ++j) issue(j, j);
         pending = (1u << pre) - 1u;
@@ -458,13 +457,20 @@ __global__ void __launch_bounds__(kWarps * 32)
             pending &= ~(1u << s);
             const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
             uint8_t* sK = ring + s * STAGE;
+            // Generic-proxy writes into the stage (the new token's row, zeroed
+            // rows past the end) must be ordered before the next TMA write to
+            // it; plain reads need no fence (their values are consumed first).
+            bool wrote = GQA && valid < kPageSize;
             if constexpr (FUSED) {
                 // the issue side has not moved past this page's id window
-                if (en.chunk == en.n_chunks - 1 && j == np - 1)
-                    put_new_token<D>(p, en, g, __shfl_sync(0xffffffffu, pid_cur, j & 31), sK, sK + TILE, lane);
+                if (en.chunk == en.n_chunks - 1 && j == np - 1) {
+                    int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
+                    put_new_token<D>(p, en, g, (pid < 0 || pid >= p.num_pages) ? 0 : pid, sK, sK + TILE, lane);
+                    wrote = true;
+                }
             }
             comp.page(sK, sK + TILE, ring_s + s * STAGE, ring_s + s * STAGE + TILE, valid, p.scale_log2, lane);
-            fence_proxy_async_smem();
+            if (wrote) fence_proxy_async_smem();
             __syncwarp();
             if (j + R < np) {
                 issue(j + R, s);
@@ -473,7 +479,7 @@ __global__ void __launch_bounds__(kWarps * 32)
         }
         if (!ok) break;
         comp.finish(p, en, g, lane);
-        if (lane == 0) item = (int)atomicAdd(&p.queue[0], 1u);
+        if (lane == 0) item = n_warps + (int)atomicAdd(&p.queue[0], 1u);
         item = __shfl_sync(0xffffffffu, item, 0);
     }
 
@@ -574,7 +580,7 @@ template <int D, bool GQA, bool FUSED>
 cudaError_t prepare_variant()
 {
     static cudaError_t status = cudaFuncSetAttribute(decode_kernel<D, GQA, FUSED>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, Geo<D>::kSmem);
+                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, Geo<D, GQA>::kSmem);
     return status;
 }
 
@@ -585,9 +591,9 @@ cudaError_t variant_info(DecodeVariant* v)
     if (e == cudaSuccess) e = prepare_variant<D, GQA, true>();
     if (e != cudaSuccess) return e;
     v->warps = kWarps;
-    v->smem_bytes = Geo<D>::kSmem;
+    v->smem_bytes = Geo<D, GQA>::kSmem;
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v->ctas_per_sm, decode_kernel<D, GQA, false>, kWarps * 32,
-                                                         Geo<D>::kSmem);
+                                                         Geo<D, GQA>::kSmem);
 }
 
 template <int D, bool GQA>
@@ -597,7 +603,7 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
     if (!fused) {
         cudaError_t e = prepare_variant<D, GQA, false>();
         if (e != cudaSuccess) return e;
-        decode_kernel<D, GQA, false><<<grid, kWarps * 32, Geo<D>::kSmem, st>>>(tk, tv, p);
+        decode_kernel<D, GQA, false><<<grid, kWarps * 32, Geo<D, GQA>::kSmem, st>>>(tk, tv, p);
         return cudaGetLastError();
     }
     cudaError_t e = prepare_variant<D, GQA, true>();
@@ -605,7 +611,7 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(kWarps * 32);
-    cfg.dynamicSmemBytes = Geo<D>::kSmem;
+    cfg.dynamicSmemBytes = Geo<D, GQA>::kSmem;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

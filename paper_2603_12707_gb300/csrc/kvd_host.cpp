@@ -54,6 +54,21 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 void kvd::set_last_error(const char* msg) { g_last_error = msg; }
 
+CUresult kvd::encode_tile_map(void* encode_fn, CUtensorMap* map, void* k_pool, int64_t rows, int D,
+                              int64_t v_stride_bytes)
+{
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(encode_fn);
+    // dims (innermost first): 64 columns, rows, D/64 column blocks, [K, V]
+    cuuint64_t gdim[4] = {64, (cuuint64_t)rows, (cuuint64_t)(D / 64), 2};
+    cuuint64_t gstride[3] = {(cuuint64_t)D * sizeof(uint16_t), 128, (cuuint64_t)v_stride_bytes};
+    cuuint32_t box[4] = {64, (cuuint32_t)kPageSize, (cuuint32_t)(D / 64), 2};
+    cuuint32_t estride[4] = {1, 1, 1, 1};
+    const cuuint32_t rank = v_stride_bytes > 0 ? 4 : 3;
+    return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, k_pool, gdim, gstride, box, estride,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 struct kv_cache {
     kvc_config cfg{};
     bool host_only = false;
@@ -82,10 +97,13 @@ struct kv_cache {
     int32_t* err = nullptr;
     PlanEntry* plan = nullptr;
     int64_t plan_cap = 0;
+    int32_t* item_pages = nullptr;              // [entries][page_stride]
+    int64_t item_pages_cap = 0;
+    int32_t page_stride = 0;
     float* part_o = nullptr;
     float2* part_ml = nullptr;
     int64_t slot_cap = 0;
-    std::vector<CUtensorMap> tmaps;             // [L][2]: K, V
+    std::vector<CUtensorMap> tmaps;             // [L]: K and V of a layer
 
     // current step
     bool step_active = false;
@@ -151,8 +169,16 @@ int32_t auto_item_pages(const kv_cache* c, int64_t total_units)
     return (int32_t)std::min<int64_t>(128, std::max<int64_t>(2, T));
 }
 
-int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, cudaStream_t st)
+int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, int64_t page_ids, cudaStream_t st)
 {
+    if (page_ids > c->item_pages_cap) {
+        const int64_t cap = std::max<int64_t>(page_ids, c->item_pages_cap + c->item_pages_cap / 2);
+        if (c->item_pages) KVD_CUDA(cudaFreeAsync(c->item_pages, st));
+        c->item_pages = nullptr;
+        c->item_pages_cap = 0;
+        KVD_CUDA(cudaMallocAsync((void**)&c->item_pages, (size_t)cap * sizeof(int32_t), st));
+        c->item_pages_cap = cap;
+    }
     if (entries > c->plan_cap) {
         const int64_t cap = std::max<int64_t>(entries, c->plan_cap + c->plan_cap / 2);
         if (c->plan) KVD_CUDA(cudaFreeAsync(c->plan, st));
@@ -185,6 +211,7 @@ void release_device(kv_cache* c)
     cudaFree(c->queue);
     cudaFree(c->err);
     cudaFree(c->plan);
+    cudaFree(c->item_pages);
     cudaFree(c->part_o);
     cudaFree(c->part_ml);
 }
@@ -265,25 +292,18 @@ int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
         KVD_CUDA_C(cudaMemsetAsync(c->err, 0, sizeof(int32_t), st));
 #undef KVD_CUDA_C
 
-        // One 2-D view per layer pool: rows = (page * H_kv + head) * P + slot,
-        // D bf16 columns; tiles are boxes of 16 rows x 64 columns, 128-byte swizzle.
-        c->tmaps.resize(2 * (size_t)k.num_layers);
+        // One TMA view per layer covering its K and V pools: a page's
+        // (page, head) tiles of K and V arrive with a single load.
+        c->tmaps.resize((size_t)k.num_layers);
         for (int l = 0; l < k.num_layers; ++l) {
-            for (int kv = 0; kv < 2; ++kv) {
-                void* base = kv ? c->v_pool(l) : c->k_pool(l);
-                cuuint64_t gdim[2] = {(cuuint64_t)k.head_dim, (cuuint64_t)(k.num_pages * k.num_kv_heads * kPageSize)};
-                cuuint64_t gstride[1] = {(cuuint64_t)k.head_dim * sizeof(uint16_t)};
-                cuuint32_t box[2] = {64, (cuuint32_t)kPageSize};
-                cuuint32_t estride[2] = {1, 1};
-                CUresult r = encode(&c->tmaps[2 * l + kv], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, gdim, gstride,
-                                    box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-                if (r != CUDA_SUCCESS) {
-                    release_device(c);
-                    delete c;
-                    return fail(KVC_ERR_CUDA, "kv_cache_create: cuTensorMapEncodeTiled failed (" +
-                                                  std::to_string((int)r) + ")");
-                }
+            const int64_t v_stride = (int64_t)((char*)c->v_pool(l) - (char*)c->k_pool(l));
+            CUresult r = encode_tile_map(reinterpret_cast<void*>(encode), &c->tmaps[l], c->k_pool(l),
+                                         k.num_pages * k.num_kv_heads * kPageSize, k.head_dim, v_stride);
+            if (r != CUDA_SUCCESS) {
+                release_device(c);
+                delete c;
+                return fail(KVC_ERR_CUDA, "kv_cache_create: cuTensorMapEncodeTiled failed (" + std::to_string((int)r) +
+                                              ")");
             }
         }
     }
@@ -500,14 +520,17 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     }
     const int32_t T = c->split_override ? c->split_override : auto_item_pages(c, total_units);
     int64_t entries = 0;
+    int32_t stride = 1;
     bool split = false;
     for (int32_t b = 0; b < batch; ++b) {
         const int nch = row_chunks(np_after[b], T);
         entries += nch;
         split = split || nch > 1;
+        stride = std::max(stride, (np_after[b] + nch - 1) / nch);
     }
     if (!c->host_only)
-        if (int rc = grow_scratch(c, entries, entries * c->cfg.num_kv_heads, static_cast<cudaStream_t>(stream)))
+        if (int rc = grow_scratch(c, entries, entries * c->cfg.num_kv_heads, entries * stride,
+                                  static_cast<cudaStream_t>(stream)))
             return rc;
 
     // Host mirror: every sequence of the batch gets position len.
@@ -553,9 +576,12 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
             pa.build = (b0 + n == batch) ? 1 : 0;
             KVD_CUDA(launch_step(patch, pa, st));
         }
+        KVD_CUDA(launch_gather_pages(c->plan, (int32_t)entries, c->page_table(), c->cfg.max_pages_per_seq,
+                                     c->item_pages, stride, c->num_sms, st));
     }
     c->step_active = true;
     c->step_split = split;
+    c->page_stride = stride;
     c->step_batch = batch;
     c->step_entries = (int32_t)entries;
     return KVC_OK;
@@ -614,6 +640,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.part_o = c->part_o;
     p.part_ml = c->part_ml;
     p.rows = c->rows;
+    p.item_pages = c->item_pages;
+    p.page_stride = c->page_stride;
     p.batch = batch;
     // A fused launch may start while the previous one drains, so consecutive
     // fused launches use different work counters.
@@ -633,8 +661,9 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     const int64_t resident = (int64_t)c->num_sms * std::max(1, c->variant.ctas_per_sm);
     const int64_t want = (p.n_items + c->variant.warps - 1) / c->variant.warps;
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
-    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[2 * layer], c->tmaps[2 * layer + 1],
-                           p, static_cast<cudaStream_t>(stream)));
+    p.kv_map = 1;
+    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[layer], c->tmaps[layer], p,
+                           static_cast<cudaStream_t>(stream)));
     if (c->step_split)
         KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->num_sms, p, static_cast<cudaStream_t>(stream)));
     if (fused) ++c->fused_launches;

@@ -111,6 +111,8 @@ struct DecodeParams {
     float* part_o;            // [slots][G][D]
     float2* part_ml;          // [slots][G]  (running max in log2 units, sum)
     const int2* rows;         // [batch]: (first partial slot, items) per batch row
+    const int32_t* item_pages;// [entries][page_stride]: page ids of each plan entry's pages
+    int32_t page_stride;
     int32_t batch;
     uint32_t* queue;          // [0] next item, [1] warps finished
     int32_t* err;
@@ -125,7 +127,18 @@ struct DecodeParams {
     const uint16_t* v_new;
     uint16_t* pool_k;         // this layer's pools [num_pages][H_kv][P][D]
     uint16_t* pool_v;
+    // 1: the first tensor map covers K and V (one 4-D load per page); 0: two
+    // 3-D maps, K and V.
+    int32_t kv_map;
 };
+
+// TMA view of a (page, head) tile: box {64 columns, 16 rows, D/64 column
+// halves} of a pool whose rows are D bf16 (row index (page*H_kv + head)*16 +
+// slot), 128-byte swizzle; with v_stride_bytes > 0 a fourth dimension of 2
+// steps from the K pool to the V pool.  Shared-memory image: [K, V][half]
+// [16 rows][128 B].  `encode` is cuTensorMapEncodeTiled.
+CUresult encode_tile_map(void* encode_fn, CUtensorMap* map, void* k_pool, int64_t rows, int D,
+                         int64_t v_stride_bytes);
 
 // Message returned by kv_last_error() on the calling thread.
 void set_last_error(const char* msg);
@@ -134,6 +147,10 @@ void set_last_error(const char* msg);
 cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st);
 cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, cudaStream_t st);
 cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
+// Copy each plan entry's page ids from the page table into item_pages
+// ([entries][stride]), so the decode kernel reads them alongside the entry.
+cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
+                                int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
 
 // Decode attention: variant chosen by (D, G == 1).

@@ -172,7 +172,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     int64_t T = std::min<int64_t>(128, std::max<int64_t>(2, (total_pages * num_kv_heads + 3 * warps - 1) / (3 * warps)));
     int64_t entries = 0;
     bool split_rows = false;
-    size_t off_o = 0, off_ml = 0, off_rows = 0, off_q = 0, off_err = 0, need = 0;
+    int stride = 1;
+    size_t off_pages = 0, off_o = 0, off_ml = 0, off_rows = 0, off_q = 0, off_err = 0, need = 0;
     for (;; T *= 2) {
         entries = 0;
         int64_t split_items = 0;   // only rows cut into several items keep partials
@@ -183,7 +184,14 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
         }
         split_rows = split_items > 0;
         const int64_t slots = split_items * num_kv_heads;
-        off_o = round256((size_t)entries * sizeof(PlanEntry));
+        stride = 1;
+        for (int b = 0; b < batch; ++b) {
+            const int np = (lens[b] + kPageSize - 1) / kPageSize;
+            const int nch = row_chunks(np, (int)T);
+            stride = std::max(stride, (np + nch - 1) / nch);
+        }
+        off_pages = round256((size_t)entries * sizeof(PlanEntry));
+        off_o = round256(off_pages + (size_t)entries * stride * sizeof(int32_t));
         off_ml = round256(off_o + (size_t)slots * G * head_dim * sizeof(float));
         off_rows = round256(off_ml + (size_t)slots * G * sizeof(float2));
         off_q = round256(off_rows + (size_t)batch * sizeof(int2));
@@ -199,13 +207,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     if (!encode) return fail(KVC_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
     CUtensorMap maps[2];
     for (int kv = 0; kv < 2; ++kv) {
-        cuuint64_t gdim[2] = {(cuuint64_t)head_dim, (cuuint64_t)(num_pages * num_kv_heads * kPageSize)};
-        cuuint64_t gstride[1] = {(cuuint64_t)head_dim * sizeof(uint16_t)};
-        cuuint32_t box[2] = {64, (cuuint32_t)kPageSize};
-        cuuint32_t estride[2] = {1, 1};
-        CUresult r = encode(&maps[kv], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(kv ? v_pool : k_pool),
-                            gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        CUresult r = encode_tile_map(reinterpret_cast<void*>(encode), &maps[kv], const_cast<void*>(kv ? v_pool : k_pool),
+                                     num_pages * num_kv_heads * kPageSize, head_dim, 0);
         if (r != CUDA_SUCCESS) return fail(KVC_ERR_INVALID, "cuTensorMapEncodeTiled rejected the pools");
     }
 
@@ -233,6 +236,11 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     }
     noalloc_plan_kernel<<<1, 1024, 0, st>>>(pa);
     if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
+    int32_t* item_pages = reinterpret_cast<int32_t*>(scratch + off_pages);
+    if (cudaError_t e = launch_gather_pages(pa.plan, (int32_t)entries, page_table, max_pages, item_pages, stride,
+                                            num_sms, st);
+        e != cudaSuccess)
+        return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
 
     const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)head_dim);
     DecodeParams p;
@@ -243,6 +251,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.part_o = reinterpret_cast<float*>(scratch + off_o);
     p.part_ml = reinterpret_cast<float2*>(scratch + off_ml);
     p.rows = pa.rows;
+    p.item_pages = item_pages;
+    p.page_stride = stride;
     p.batch = batch;
     p.queue = pa.queue;
     p.err = pa.err;
@@ -253,6 +263,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.G = G;
     p.max_pages = max_pages;
     p.scale_log2 = scale * 1.4426950408889634f;
+    p.kv_map = 0;
     p.k_new = p.v_new = nullptr;
     p.pool_k = p.pool_v = nullptr;
     const int64_t resident = (int64_t)num_sms * std::max(1, var.ctas_per_sm);
