@@ -53,29 +53,25 @@ __device__ __forceinline__ uint32_t swz(int r, int c)
     return (uint32_t)((c >> 3) * 2048 + r * 128 + (((c & 7) ^ (r & 7)) << 4));
 }
 
-__device__ __forceinline__ float dot8(const uint4& k, const float (&q)[8])
+// q . k over one 16-byte chunk (8 dims): k bf16, q as four f32 pairs.
+__device__ __forceinline__ float dot8(const uint4& k, const uint64_t (&q2)[4])
 {
-    float s = bf16lo(k.x) * q[0];
-    s = fmaf(bf16hi(k.x), q[1], s);
-    s = fmaf(bf16lo(k.y), q[2], s);
-    s = fmaf(bf16hi(k.y), q[3], s);
-    s = fmaf(bf16lo(k.z), q[4], s);
-    s = fmaf(bf16hi(k.z), q[5], s);
-    s = fmaf(bf16lo(k.w), q[6], s);
-    s = fmaf(bf16hi(k.w), q[7], s);
-    return s;
+    uint64_t acc = f2_fma(q2[0], bf16x2_to_f2(k.x), 0ull);
+    acc = f2_fma(q2[1], bf16x2_to_f2(k.y), acc);
+    acc = f2_fma(q2[2], bf16x2_to_f2(k.z), acc);
+    acc = f2_fma(q2[3], bf16x2_to_f2(k.w), acc);
+    float lo, hi;
+    f2_unpack(acc, lo, hi);
+    return lo + hi;
 }
 
-__device__ __forceinline__ void axpy8(float (&o)[8], float p, const uint4& v)
+// o += p * v over one 16-byte chunk, o as four f32 pairs.
+__device__ __forceinline__ void axpy8(uint64_t (&o2)[4], uint64_t p2, const uint4& v)
 {
-    o[0] = fmaf(p, bf16lo(v.x), o[0]);
-    o[1] = fmaf(p, bf16hi(v.x), o[1]);
-    o[2] = fmaf(p, bf16lo(v.y), o[2]);
-    o[3] = fmaf(p, bf16hi(v.y), o[3]);
-    o[4] = fmaf(p, bf16lo(v.z), o[4]);
-    o[5] = fmaf(p, bf16hi(v.z), o[5]);
-    o[6] = fmaf(p, bf16lo(v.w), o[6]);
-    o[7] = fmaf(p, bf16hi(v.w), o[7]);
+    o2[0] = f2_fma(p2, bf16x2_to_f2(v.x), o2[0]);
+    o2[1] = f2_fma(p2, bf16x2_to_f2(v.y), o2[1]);
+    o2[2] = f2_fma(p2, bf16x2_to_f2(v.z), o2[2]);
+    o2[3] = f2_fma(p2, bf16x2_to_f2(v.w), o2[3]);
 }
 
 // ------------------------------------------------------------ MHA, CUDA cores
@@ -87,22 +83,23 @@ struct MhaCompute {
     static constexpr int IT = kPageSize / TPI;
     static constexpr int LOG_IT = (IT == 8) ? 3 : (IT == 4 ? 2 : 1);
     int c, tsub;
-    float qf[8];
-    float m, l, o[8];
+    uint64_t q2[4];          // q of this lane's chunk as f32 pairs
+    float m, l;
+    uint64_t o2[4];          // unnormalised output of this lane's chunk, f32 pairs
 
     __device__ __forceinline__ void start(const DecodeParams& p, const PlanEntry& en, int g, int lane)
     {
         c = lane % CH;
         tsub = lane / CH;
         const uint4 qq = *reinterpret_cast<const uint4*>(p.q + ((int64_t)en.b * p.H_q + g) * D + c * 8);
-        qf[0] = bf16lo(qq.x); qf[1] = bf16hi(qq.x);
-        qf[2] = bf16lo(qq.y); qf[3] = bf16hi(qq.y);
-        qf[4] = bf16lo(qq.z); qf[5] = bf16hi(qq.z);
-        qf[6] = bf16lo(qq.w); qf[7] = bf16hi(qq.w);
+        q2[0] = bf16x2_to_f2(qq.x);
+        q2[1] = bf16x2_to_f2(qq.y);
+        q2[2] = bf16x2_to_f2(qq.z);
+        q2[3] = bf16x2_to_f2(qq.w);
         m = -INFINITY;
         l = 0.f;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) o[k] = 0.f;
+        for (int k = 0; k < 4; ++k) o2[k] = 0ull;
     }
 
     __device__ __forceinline__ void page(uint8_t* sK, uint8_t* sV, uint32_t, uint32_t, int valid,
@@ -112,7 +109,7 @@ struct MhaCompute {
 #pragma unroll
         for (int i = 0; i < IT; ++i) {
             const uint4 kv = *reinterpret_cast<const uint4*>(sK + swz(i * TPI + tsub, c));
-            part[i] = dot8(kv, qf);
+            part[i] = dot8(kv, q2);
         }
         // Reduce-scatter over the CH lanes of a row: afterwards lane c holds
         // token (c >> 1) * TPI + tsub, summed over all chunks.
@@ -139,15 +136,16 @@ struct MhaCompute {
         const float pe = ex2(sc - mn);
         l = fmaf(l, alpha, (c & 1) ? 0.f : pe);
         m = mn;
+        const uint64_t a2 = f2_pack(alpha, alpha);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) o[k] *= alpha;
+        for (int k = 0; k < 4; ++k) o2[k] = f2_fma(o2[k], a2, 0ull);
 #pragma unroll
         for (int i = 0; i < IT; ++i) {
             const float pt = __shfl_sync(0xffffffffu, pe, tsub * CH + 2 * i);
             const int t = i * TPI + tsub;
             if (t < valid) {   // rows past the end may hold anything
                 const uint4 vv = *reinterpret_cast<const uint4*>(sV + swz(t, c));
-                axpy8(o, pt, vv);
+                axpy8(o2, f2_pack(pt, pt), vv);
             }
         }
     }
@@ -156,6 +154,9 @@ struct MhaCompute {
     // row; the merge pass combines them).
     __device__ __forceinline__ void finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
     {
+        float o[8];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) f2_unpack(o2[k], o[2 * k], o[2 * k + 1]);
 #pragma unroll
         for (int mask = CH; mask < 32; mask <<= 1)
 #pragma unroll
@@ -501,12 +502,13 @@ __global__ void __launch_bounds__(kWarps * 32)
     }
 }
 
-// Second pass.  Warp w handles (row b, query head h) = (w / H_q, w % H_q) of
-// a split row: lane c < n_chunks holds item c's (m, l); the weights
-// 2^(m_c - M) / sum_c 2^(m_c - M) l_c stay in registers and are broadcast
-// while the lanes (D/32 dims each) accumulate the items' o, eight items in
-// flight at a time.
+// Second pass.  A split row's (row b, query head h) is merged by SPLIT warps,
+// each owning D/SPLIT dims: lane c < n_chunks holds item c's (m, l); the
+// weights 2^(m_c - M) / sum_c 2^(m_c - M) l_c stay in registers and are
+// broadcast while the lanes (D/SPLIT/32 dims each) accumulate the items' o,
+// sixteen items in flight at a time.
 constexpr int kMergeWarps = 4;
+constexpr int kMergeSplit = 2;
 
 template <int D>
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodeParams p, int pdl)
@@ -515,11 +517,15 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
         griddep_launch_dependents();   // the next layer may start streaming now
         griddep_wait();                // the split pass of this layer is complete
     }
-    constexpr int PER = D / 32;
+    constexpr int DW = D / kMergeSplit;   // dims per warp
+    constexpr int PER = DW / 32;          // dims per lane
+    constexpr int U = 16;
     const int lane = threadIdx.x & 31;
-    const int total = p.batch * p.H_q;
+    const int total = p.batch * p.H_q * kMergeSplit;
     for (int w = blockIdx.x * kMergeWarps + (threadIdx.x >> 5); w < total; w += gridDim.x * kMergeWarps) {
-        const int b = w / p.H_q, h = w - b * p.H_q;
+        const int part = w % kMergeSplit;
+        const int bh = w / kMergeSplit;
+        const int b = bh / p.H_q, h = bh - b * p.H_q;
         const int2 row = p.rows[b];
         const int nch = row.y;
         if (nch <= 1) continue;
@@ -539,39 +545,36 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
 #pragma unroll
         for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
         const float wgt = e / L;
+        const int d0 = part * DW + lane * PER;
         float acc[PER];
 #pragma unroll
         for (int k = 0; k < PER; ++k) acc[k] = 0.f;
-        for (int c0 = 0; c0 < nch; c0 += 8) {
-            float v[8][PER];
+        for (int c0 = 0; c0 < nch; c0 += U) {
+            float v[U][PER];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < U; ++u) {
                 const int c = c0 + u;
-                const float* po = p.part_o + slot(c < nch ? c : 0) * D + lane * PER;
-                if constexpr (PER == 4) {
-                    const float4 t = __ldcg(reinterpret_cast<const float4*>(po));
-                    v[u][0] = t.x; v[u][1] = t.y; v[u][2] = t.z; v[u][3] = t.w;
-                } else {
+                const float* po = p.part_o + slot(c < nch ? c : 0) * D + d0;
+                if constexpr (PER == 2) {
                     const float2 t = __ldcg(reinterpret_cast<const float2*>(po));
                     v[u][0] = t.x; v[u][1] = t.y;
+                } else {
+                    v[u][0] = __ldcg(po);
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 8; ++u) {
+            for (int u = 0; u < U; ++u) {
                 const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
                 if (c0 + u < nch)
 #pragma unroll
                     for (int k = 0; k < PER; ++k) acc[k] = fmaf(wc, v[u][k], acc[k]);
             }
         }
-        uint16_t* orow = p.out + ((int64_t)b * p.H_q + h) * D + lane * PER;
-        if constexpr (PER == 4) {
-            uint2 o;
-            o.x = pack_bf16(acc[0], acc[1]);
-            o.y = pack_bf16(acc[2], acc[3]);
-            *reinterpret_cast<uint2*>(orow) = o;
-        } else {
+        uint16_t* orow = p.out + ((int64_t)b * p.H_q + h) * D + d0;
+        if constexpr (PER == 2) {
             *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0], acc[1]);
+        } else {
+            orow[0] = (uint16_t)(pack_bf16(acc[0], 0.f) & 0xffffu);
         }
     }
 }
@@ -625,7 +628,7 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
 
 cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st)
 {
-    const int64_t warps = (int64_t)p.batch * p.H_q;
+    const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
                                                                    (int64_t)num_sms * 16));
     cudaLaunchConfig_t cfg = {};

@@ -171,6 +171,33 @@ __device__ __forceinline__ float ex2(float x)
 __device__ __forceinline__ float bf16lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
+// Packed pairs of f32 (sm_100 family): one 64-bit register, two lanes.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+// d = a * b + c on both lanes, round to nearest.
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+// Two bf16 in one 32-bit word -> the f32 pair (exact).
+__device__ __forceinline__ uint64_t bf16x2_to_f2(uint32_t u)
+{
+    return f2_pack(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
 // Round two f32 to bf16 (nearest even) and pack: `lo` in bits 0-15.
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
