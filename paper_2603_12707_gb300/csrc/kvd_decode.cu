@@ -491,9 +491,10 @@ __global__ void __launch_bounds__(kWarps * 32)
         if (pending & (1u << s)) mbar_wait_bounded(smem_addr(&bars[s]), (phase >> s) & 1u, kWaitLimitNs);
     __syncwarp();
 
-    // The last warp out resets the work counter for the next launch.
-    if (lane == 31) {
-        __threadfence();
+    // The last warp out resets the work counter for the next launch.  No
+    // fence: every warp consumed the value of its last counter fetch before
+    // getting here, so all fetches are performed before the reset.
+    if (lane == 0) {
         const uint32_t total = gridDim.x * kWarps;
         if (atomicAdd(&p.queue[1], 1u) == total - 1) {
             p.queue[0] = 0;
