@@ -243,6 +243,7 @@ def run_gpu(args, rank, world):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
+    launches0 = sess.query().kernel_launches
     with ClockSampler(gpu_smi_id(torch, dev)) as clocks:
         with torch.cuda.stream(stream):
             start.record(stream)
@@ -267,6 +268,7 @@ def run_gpu(args, rank, world):
         attn_bytes.append(a if args.unfused else a + p)   # the fused kernel also writes the new K/V
     st = sess.query()
     assert st.device_error == 0, st.device_error
+    timed_launches = st.kernel_launches - launches0
 
     # ---- end to end: host inputs -> device -> host outputs, every step
     e2e = None
@@ -315,6 +317,7 @@ def run_gpu(args, rank, world):
 
     sess.close()
     return {"ms": ms, "attn_ms": attn_ms, "step_bytes": step_bytes, "attn_bytes": attn_bytes,
+            "launches": timed_launches,
             "clocks": clocks.summary(), "e2e": e2e, "cfg": cfg, "L": L}
 
 
@@ -413,7 +416,7 @@ def main():
                      "traffic": (traffic["dram_bytes_per_launch_full"] if traffic else None),
                      "algorithmic_bytes_per_launch": int(attn_bytes), "avg_launch_ms": round(attn_ms, 4)},
         "clocks": r["clocks"],
-        "gpu_launches": args.steps * (1 + (2 if args.unfused else 1) * L),
+        "gpu_launches": r["launches"],
         "step_kernels": "kv_begin_step + per layer " + ("kv_append, decode_attention" if args.unfused
                                                           else "decode_attention_append (fused, PDL)"),
     }

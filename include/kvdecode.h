@@ -88,6 +88,7 @@ typedef struct kvc_stats {
     int64_t free_pages;
     int32_t live_seqs;
     int32_t device_error;       /* KVC_DEVERR_* bits found by kernels so far             */
+    int64_t kernel_launches;    /* kernels this cache has launched since creation         */
 } kvc_stats;
 
 typedef struct kv_cache kv_cache; /* opaque */

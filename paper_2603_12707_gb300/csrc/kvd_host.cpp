@@ -94,6 +94,7 @@ struct kv_cache {
     int2* rows = nullptr;                       // per batch row: (first partial slot, items)
     uint32_t* queue = nullptr;                  // two (next item, warps done) counter pairs
     uint32_t fused_launches = 0;                // fused launches alternate counter pairs
+    int64_t launches = 0;                       // kernels launched (reported by kv_cache_query)
     int32_t* err = nullptr;
     PlanEntry* plan = nullptr;
     int64_t plan_cap = 0;
@@ -154,6 +155,7 @@ int push_updates(kv_cache* c, const std::vector<int32_t>& idx, const std::vector
         std::memcpy(s.idx, idx.data() + off, n * sizeof(int32_t));
         std::memcpy(s.val, val.data() + off, n * sizeof(int32_t));
         KVD_CUDA(launch_scatter_i32(c->meta, s, st));
+        ++c->launches;
     }
     return KVC_OK;
 }
@@ -349,6 +351,7 @@ int kv_cache_query(kv_cache* c, kvc_stats* s)
     s->pool_bytes = c->host_only ? 0 : (int64_t)(2 * (size_t)k.num_layers * c->layer_elems * sizeof(uint16_t));
     s->live_seqs = c->live;
     s->device_error = 0;
+    s->kernel_launches = c->launches;
     if (c->host_only) return KVC_OK;
     KVD_CUDA(cudaDeviceSynchronize());
     KVD_CUDA(cudaMemcpy(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost));
@@ -474,6 +477,7 @@ static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq,
     a.to_pool = to_pool;
     a.err = c->err;
     KVD_CUDA(launch_token_copy(a, static_cast<cudaStream_t>(stream)));
+    ++c->launches;
     return KVC_OK;
 }
 
@@ -575,9 +579,11 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
             }
             pa.build = (b0 + n == batch) ? 1 : 0;
             KVD_CUDA(launch_step(patch, pa, st));
+            ++c->launches;
         }
         KVD_CUDA(launch_gather_pages(c->plan, (int32_t)entries, c->page_table(), c->cfg.max_pages_per_seq,
                                      c->item_pages, stride, c->num_sms, st));
+        ++c->launches;
     }
     c->step_active = true;
     c->step_split = split;
@@ -617,6 +623,7 @@ int kv_append(kv_cache* c, int32_t layer, int32_t batch, const void* k_new, cons
     a.max_pages = c->cfg.max_pages_per_seq;
     a.err = c->err;
     KVD_CUDA(launch_append(a, static_cast<cudaStream_t>(stream)));
+    ++c->launches;
     return KVC_OK;
 }
 
@@ -664,8 +671,11 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.kv_map = 1;
     KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[layer], c->tmaps[layer], p,
                            static_cast<cudaStream_t>(stream)));
-    if (c->step_split)
+    ++c->launches;
+    if (c->step_split) {
         KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->num_sms, p, static_cast<cudaStream_t>(stream)));
+        ++c->launches;
+    }
     if (fused) ++c->fused_launches;
     return KVC_OK;
 }

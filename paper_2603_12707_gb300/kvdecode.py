@@ -49,7 +49,8 @@ class kvc_config(ctypes.Structure):
 class kvc_stats(ctypes.Structure):
     _fields_ = [("kv_bytes_allocated", ctypes.c_int64), ("pool_bytes", ctypes.c_int64),
                 ("pages_in_use", ctypes.c_int64), ("free_pages", ctypes.c_int64),
-                ("live_seqs", ctypes.c_int32), ("device_error", ctypes.c_int32)]
+                ("live_seqs", ctypes.c_int32), ("device_error", ctypes.c_int32),
+                ("kernel_launches", ctypes.c_int64)]
 
 
 _lib = None
