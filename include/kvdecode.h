@@ -243,6 +243,13 @@ KVC_API int decode_attention_noalloc(const void *k_pool, const void *v_pool, int
                                      const int32_t *lens, const void *q, void *out,
                                      float softmax_scale, int32_t *device_error, void *stream);
 
+/* Diagnostics: one warp runs the bounded shared-memory wait that every
+ * pipeline wait of the decode kernels uses, on a barrier that nothing ever
+ * completes, and writes 1 to *status (device int32) when the wait gave up
+ * after limit_ns nanoseconds (0 < limit_ns <= 2e9), 0 if it completed.  The
+ * GPU context stays usable afterwards.  Asynchronous on `stream`. */
+KVC_API int kv_selftest_wait_timeout(int64_t limit_ns, int32_t *status, void *stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 KVC_API const char *kv_last_error(void);
 

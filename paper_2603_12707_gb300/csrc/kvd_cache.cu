@@ -3,6 +3,7 @@
 #include <algorithm>
 
 #include "kvd_internal.h"
+#include "kvd_ptx.cuh"
 
 namespace kvd {
 
@@ -162,7 +163,28 @@ __global__ void gather_pages_kernel(const PlanEntry* plan, int32_t entries, cons
     }
 }
 
+// One warp waits, with the decode kernel's bounded wait, on an mbarrier that
+// nothing arrives on; status = 1 when the wait gave up, 0 if it completed.
+__global__ void wait_timeout_kernel(uint64_t limit_ns, int32_t* status)
+{
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_addr(&bar), 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    const bool done = mbar_wait_bounded(smem_addr(&bar), 0, limit_ns);
+    if (threadIdx.x == 0) *status = __all_sync(0xffffffffu, done) ? 0 : 1;
+    else (void)__all_sync(0xffffffffu, done);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_timeout_check(uint64_t limit_ns, int32_t* status, cudaStream_t st)
+{
+    wait_timeout_kernel<<<1, 32, 0, st>>>(limit_ns, status);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
                                 int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st)

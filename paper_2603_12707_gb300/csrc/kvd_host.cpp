@@ -693,4 +693,12 @@ int decode_attention_append(kv_cache* c, int32_t layer, int32_t batch, const voi
     return launch_attention(c, "decode_attention_append", layer, batch, q, k_new, v_new, out, softmax_scale, stream);
 }
 
+int kv_selftest_wait_timeout(int64_t limit_ns, int32_t* status, void* stream)
+{
+    if (!status || limit_ns <= 0 || limit_ns > 2000000000ll)
+        return fail(KVC_ERR_INVALID, "kv_selftest_wait_timeout: status must be non-null, 0 < limit_ns <= 2e9");
+    KVD_CUDA(launch_wait_timeout_check((uint64_t)limit_ns, status, static_cast<cudaStream_t>(stream)));
+    return KVC_OK;
+}
+
 }  // extern "C"

@@ -152,6 +152,7 @@ cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
 cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
                                 int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
+cudaError_t launch_wait_timeout_check(uint64_t limit_ns, int32_t* status, cudaStream_t st);
 
 // Decode attention: variant chosen by (D, G == 1).
 struct DecodeVariant {

@@ -74,6 +74,7 @@ _SIGS = {
     "kv_append": [_P, _I32, _I32, _P, _P, _P],
     "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
     "decode_attention_append": [_P, _I32, _I32, _P, _P, _P, _P, ctypes.c_float, _P],
+    "kv_selftest_wait_timeout": [_I64, _P, _P],
     "decode_attention_noalloc": [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _I32, _P, _P, _P,
                                  ctypes.c_float, _P, _P],
 }
@@ -224,6 +225,11 @@ def decode_attention_noalloc(k_pool, v_pool, num_pages: int, num_q_heads: int, n
                                            ctypes.addressof(arr), _ptr(q), _ptr(out), float(softmax_scale),
                                            _ptr(device_error), _stream(stream)),
            "decode_attention_noalloc")
+
+
+def kv_selftest_wait_timeout(limit_ns: int, status, stream=None):
+    _check(load().kv_selftest_wait_timeout(int(limit_ns), _ptr(status), _stream(stream)),
+           "kv_selftest_wait_timeout")
 
 
 def make_config(num_layers, num_q_heads, num_kv_heads, head_dim, num_pages, max_seqs, max_pages_per_seq,
