@@ -66,6 +66,7 @@ extern "C" {
 #define KVC_DEVERR_PAGE_RANGE 1   /* a page-table entry outside [0, num_pages) */
 #define KVC_DEVERR_WAIT_TIMEOUT 2 /* a shared-memory pipeline wait gave up      */
 #define KVC_DEVERR_SEQ_RANGE 4    /* a sequence length outside its page row     */
+#define KVC_DEVERR_OOM 8          /* a device-side step found the pool exhausted */
 
 typedef struct kvc_config {
     int32_t num_layers;        /* L: layer pools held (>= 1)                              */
@@ -104,8 +105,8 @@ typedef struct kv_cache kv_cache; /* opaque */
  * page_size != 16 or G > 8; KVC_ERR_OOM if device memory runs out. */
 KVC_API int kv_cache_create(const kvc_config *cfg, void *stream, kv_cache **out);
 
-/* Free everything the cache owns (stream-ordered on the creation stream,
- * after a device synchronisation of that stream).  NULL is accepted. */
+/* Synchronise the device, then free everything the cache owns.  NULL is
+ * accepted. */
 KVC_API int kv_cache_destroy(kv_cache *cache);
 
 /* Install the order in which free pages are handed out: order[0] first.
@@ -113,9 +114,10 @@ KVC_API int kv_cache_destroy(kv_cache *cache);
  * 0 .. num_pages-1, and no page may be in use. */
 KVC_API int kv_cache_set_page_order(kv_cache *cache, const int32_t *order, int64_t n);
 
-/* Synchronise the cache's stream and report usage and device error bits.
- * Returns KVC_ERR_PAGE_TABLE / KVC_ERR_DEVICE if device_error is non-zero
- * (the stats are filled in either way). */
+/* Synchronise the device and report usage and device error bits.  Returns
+ * KVC_ERR_PAGE_TABLE (page or length range), KVC_ERR_OOM (a device-side step
+ * ran out of pages) or KVC_ERR_DEVICE (a pipeline wait gave up) if
+ * device_error is non-zero; the stats are filled in either way. */
 KVC_API int kv_cache_query(kv_cache *cache, kvc_stats *stats);
 
 /* Device pointers of one layer's K and V pools ([num_pages][H_kv][P][d_h]
@@ -208,6 +210,35 @@ KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, cons
 KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batch, const void *q,
                                     const void *k_new, const void *v_new, void *out,
                                     float softmax_scale, void *stream);
+
+/* ------------------------------------------- graph-replayable decode step -- */
+
+/* Enable (enable = 1) or disable device-side steps.  While enabled, the free
+ * page stack also lives on the device and kv_begin_step_device performs the
+ * step's lazy allocation and split plan there, so a whole decode step
+ * (kv_begin_step_device, then per layer decode_attention_append or
+ * kv_append + decode_attention) can be captured once into a CUDA graph and
+ * replayed every step with no host work (the role CUDA graphs play in the
+ * paper's engine, Sec. 5.4).  Enabling reserves plan, page-list and partial
+ * buffers for up to max_batch sequences at the longest page-table row, and
+ * fixes the work-item size from the pages currently held.  The host
+ * allocator's view is refreshed from the device (a device synchronisation)
+ * by the next call that needs it: kv_seq_reserve, kv_seq_free, kv_seq_info,
+ * kv_begin_step, kv_cache_query, kv_write_tokens, kv_read_tokens,
+ * kv_cache_set_page_order, or kv_cache_sync. */
+KVC_API int kv_cache_device_steps(kv_cache *cache, int32_t max_batch, int32_t enable, void *stream);
+
+/* kv_begin_step with everything on the device: seq_ids is DEVICE memory
+ * ([batch] distinct live sequence ids, read when the kernel runs, so a
+ * replayed graph may change them between replays); pages come off the
+ * device free stack in batch order, exactly as kv_begin_step takes them.
+ * A pool that runs out sets KVC_DEVERR_OOM (the row keeps its length).  No
+ * host synchronisation; graph-capturable. */
+KVC_API int kv_begin_step_device(kv_cache *cache, int32_t batch, const int32_t *seq_ids, void *stream);
+
+/* Synchronise the device and refresh the host allocator's view after
+ * device-side steps. */
+KVC_API int kv_cache_sync(kv_cache *cache);
 
 /* ------------------------------------------------ allocation-free decode -- */
 

@@ -89,6 +89,78 @@ __global__ void __launch_bounds__(1024)
     }
 }
 
+// The same step on the device (graph-replayable, no host input): rows in
+// batch order reserve position len; a row whose position opens a page takes
+// the next page of the device free stack, in batch order (the same pages the
+// host allocator would hand out); then the split plan, rows in batch order.
+__global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
+{
+    __shared__ int s_top;
+    if (threadIdx.x == 0) s_top = *a.free_top;
+    __syncthreads();
+    const int top0 = s_top;
+    int carry = 0;
+    for (int base = 0; base < a.batch; base += blockDim.x) {
+        const int i = base + threadIdx.x;
+        int seq = 0, len = 0, need = 0;
+        bool ok = false;
+        if (i < a.batch) {
+            seq = a.seq_ids[i];
+            len = a.seq_len[seq];
+            ok = len >= 0 && len + 1 <= a.max_pages * kPageSize;
+            if (!ok) flag_error(a.err, 4);
+            need = (ok && len % kPageSize == 0) ? 1 : 0;
+        }
+        int total;
+        const int rank = carry + block_exclusive_scan(need, &total);
+        if (ok) {
+            int32_t page = -1;
+            if (need) {
+                const int idx = top0 - 1 - rank;
+                if (idx < 0) {
+                    flag_error(a.err, 8);   // pool exhausted
+                    ok = false;
+                } else {
+                    page = a.free_pages[idx];
+                }
+            }
+            if (ok) {
+                if (page >= 0) a.page_table[(int64_t)seq * a.max_pages + len / kPageSize] = page;
+                a.seq_len[seq] = len + 1;
+            }
+        }
+        if (i < a.batch) a.step_seq[i] = seq;
+        carry += total;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) *a.free_top = top0 - min(carry, top0);
+    carry = 0;
+    for (int base = 0; base < a.batch; base += blockDim.x) {
+        const int b = base + threadIdx.x;
+        int seq = 0, len = 0, np = 0, nch = 0;
+        if (b < a.batch) {
+            seq = a.step_seq[b];
+            len = max(1, a.seq_len[seq]);
+            np = (len + kPageSize - 1) / kPageSize;
+            nch = row_chunks(np, a.item_pages);
+        }
+        int total;
+        const int off = carry + block_exclusive_scan(nch, &total);
+        if (off + nch > a.max_entries) {
+            flag_error(a.err, 4);
+            nch = 0;
+        }
+        for (int c = 0; c < nch; ++c) {
+            int first, n;
+            chunk_range(np, nch, c, &first, &n);
+            a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
+        }
+        if (b < a.batch) a.rows[b] = make_int2(off, nch);
+        carry += total;
+    }
+    if (threadIdx.x == 0) *a.n_entries = min(carry, a.max_entries);
+}
+
 // One thread per 16-byte chunk of a [n][H_kv][D] token block.
 __global__ void token_copy_kernel(const TokenCopyArgs a)
 {
@@ -150,10 +222,12 @@ __global__ void append_kernel(const AppendArgs a)
 }
 
 // One warp per plan entry: its page ids, contiguous, at entry * stride.
-__global__ void gather_pages_kernel(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
-                                    int32_t max_pages, int32_t* item_pages, int32_t stride)
+__global__ void gather_pages_kernel(const PlanEntry* plan, int32_t entries, const int32_t* entries_dev,
+                                    const int32_t* page_table, int32_t max_pages, int32_t* item_pages,
+                                    int32_t stride)
 {
     const int lane = threadIdx.x & 31;
+    if (entries_dev) entries = min(entries, *entries_dev);
     const int warps = (gridDim.x * blockDim.x) >> 5;
     for (int e = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; e < entries; e += warps) {
         const PlanEntry en = plan[e];
@@ -186,13 +260,21 @@ cudaError_t launch_wait_timeout_check(uint64_t limit_ns, int32_t* status, cudaSt
     return cudaGetLastError();
 }
 
-cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
-                                int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st)
+cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* entries_dev,
+                                const int32_t* page_table, int32_t max_pages, int32_t* item_pages, int32_t stride,
+                                int num_sms, cudaStream_t st)
 {
     if (entries <= 0) return cudaSuccess;
     const int64_t want = ((int64_t)entries + 7) / 8;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * 8));
-    gather_pages_kernel<<<grid, 256, 0, st>>>(plan, entries, page_table, max_pages, item_pages, stride);
+    gather_pages_kernel<<<grid, 256, 0, st>>>(plan, entries, entries_dev, page_table, max_pages, item_pages,
+                                              stride);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_step_device(const StepDevArgs& a, cudaStream_t st)
+{
+    step_device_kernel<<<1, 1024, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -401,7 +401,8 @@ __global__ void __launch_bounds__(kWarps * 32)
     const int n_warps = (int)gridDim.x * kWarps;
     int item = (int)blockIdx.x * kWarps + warp;
 
-    while (item < p.n_items) {
+    const int n_items = p.n_entries_dev ? min(p.n_items, *p.n_entries_dev * p.H_kv) : p.n_items;
+    while (item < n_items) {
         const int e = item / p.H_kv;
         const int g = item - e * p.H_kv;
         // The entry's page ids sit at a fixed stride, so they load alongside

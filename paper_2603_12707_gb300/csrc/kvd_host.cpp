@@ -106,8 +106,19 @@ struct kv_cache {
     int64_t slot_cap = 0;
     std::vector<CUtensorMap> tmaps;             // [L]: K and V of a layer
 
+    // device-side steps (kv_begin_step_device): free stack on the device
+    bool dev_mode = false;                      // kv_cache_device_steps enabled
+    bool dev_dirty = false;                     // the device state moved past the host mirror
+    int32_t dev_max_batch = 0;
+    int32_t dev_item_pages = 0;
+    int32_t dev_entries_cap = 0;
+    int32_t dev_stride = 0;
+    int32_t* d_free = nullptr;                  // [num_pages]
+    int32_t* d_small = nullptr;                 // [0] free top, [1] plan entries of the step
+
     // current step
     bool step_active = false;
+    bool step_dev = false;                      // the step's plan was built on the device
     bool step_split = false;                    // some row of the step has several items
     int32_t step_batch = 0;
     int32_t step_entries = 0;
@@ -214,8 +225,50 @@ void release_device(kv_cache* c)
     cudaFree(c->err);
     cudaFree(c->plan);
     cudaFree(c->item_pages);
+    cudaFree(c->d_free);
+    cudaFree(c->d_small);
     cudaFree(c->part_o);
     cudaFree(c->part_ml);
+}
+
+// Bring the host mirror up to the device after device-side steps.
+int sync_from_device(kv_cache* c)
+{
+    if (!c->dev_dirty) return KVC_OK;
+    const kvc_config& k = c->cfg;
+    std::vector<int32_t> pt((size_t)k.max_seqs * k.max_pages_per_seq), lens((size_t)k.max_seqs);
+    int32_t small[2] = {0, 0};
+    KVD_CUDA(cudaDeviceSynchronize());
+    KVD_CUDA(cudaMemcpy(pt.data(), c->page_table(), pt.size() * sizeof(int32_t), cudaMemcpyDeviceToHost));
+    KVD_CUDA(cudaMemcpy(lens.data(), c->seq_len_dev(), lens.size() * sizeof(int32_t), cudaMemcpyDeviceToHost));
+    KVD_CUDA(cudaMemcpy(small, c->d_small, sizeof(small), cudaMemcpyDeviceToHost));
+    c->free_stack.assign((size_t)small[0], 0);
+    if (small[0] > 0)
+        KVD_CUDA(cudaMemcpy(c->free_stack.data(), c->d_free, (size_t)small[0] * sizeof(int32_t),
+                            cudaMemcpyDeviceToHost));
+    c->pages_in_use = k.num_pages - small[0];
+    for (int32_t s = 0; s < k.max_seqs; ++s) {
+        if (c->lens[s] < 0) continue;
+        c->lens[s] = lens[s];
+        const int32_t np = (lens[s] + kPageSize - 1) / kPageSize;
+        c->pages[s].assign(pt.begin() + (int64_t)s * k.max_pages_per_seq,
+                           pt.begin() + (int64_t)s * k.max_pages_per_seq + np);
+    }
+    c->dev_dirty = false;
+    return KVC_OK;
+}
+
+// After host-side allocator changes, the device free stack follows.
+int push_free_stack(kv_cache* c, cudaStream_t st)
+{
+    if (!c->dev_mode) return KVC_OK;
+    const int32_t top = (int32_t)c->free_stack.size();
+    if (top > 0)
+        KVD_CUDA(cudaMemcpyAsync(c->d_free, c->free_stack.data(), (size_t)top * sizeof(int32_t),
+                                 cudaMemcpyHostToDevice, st));
+    KVD_CUDA(cudaMemcpyAsync(c->d_small, &top, sizeof(int32_t), cudaMemcpyHostToDevice, st));
+    KVD_CUDA(cudaStreamSynchronize(st));   // the host buffers may change right after
+    return KVC_OK;
 }
 
 }  // namespace
@@ -329,6 +382,7 @@ int kv_cache_destroy(kv_cache* c)
 int kv_cache_set_page_order(kv_cache* c, const int32_t* order, int64_t n)
 {
     if (!c || !order) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: null argument");
+    if (int rc = sync_from_device(c)) return rc;
     if (n != c->cfg.num_pages) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: n must equal num_pages");
     if (c->pages_in_use) return fail(KVC_ERR_INVALID, "kv_cache_set_page_order: pages are in use");
     std::vector<uint8_t> seen((size_t)n, 0);
@@ -338,12 +392,13 @@ int kv_cache_set_page_order(kv_cache* c, const int32_t* order, int64_t n)
         seen[order[i]] = 1;
     }
     for (int64_t i = 0; i < n; ++i) c->free_stack[i] = order[n - 1 - i];
-    return KVC_OK;
+    return push_free_stack(c, nullptr);
 }
 
 int kv_cache_query(kv_cache* c, kvc_stats* s)
 {
     if (!c || !s) return fail(KVC_ERR_INVALID, "kv_cache_query: null argument");
+    if (int rc = sync_from_device(c)) return rc;
     const kvc_config& k = c->cfg;
     s->pages_in_use = c->pages_in_use;
     s->free_pages = (int64_t)c->free_stack.size();
@@ -357,6 +412,7 @@ int kv_cache_query(kv_cache* c, kvc_stats* s)
     KVD_CUDA(cudaMemcpy(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost));
     if (s->device_error & (KVC_DEVERR_PAGE_RANGE | KVC_DEVERR_SEQ_RANGE))
         return fail(KVC_ERR_PAGE_TABLE, "device found a page id or length outside its range");
+    if (s->device_error & KVC_DEVERR_OOM) return fail(KVC_ERR_OOM, "a device-side step found the page pool exhausted");
     if (s->device_error) return fail(KVC_ERR_DEVICE, "a device-side pipeline wait gave up");
     return KVC_OK;
 }
@@ -398,6 +454,7 @@ int kv_seq_create(kv_cache* c, int32_t* seq_id)
 int kv_seq_reserve(kv_cache* c, int32_t seq, int32_t n, void* stream)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_seq_reserve: null cache");
+    if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     if (n < 0) return fail(KVC_ERR_INVALID, "kv_seq_reserve: negative token count");
     const int64_t len = c->lens[seq], new_len = len + n;
@@ -415,12 +472,14 @@ int kv_seq_reserve(kv_cache* c, int32_t seq, int32_t n, void* stream)
     c->lens[seq] = (int32_t)new_len;
     idx.push_back(c->seq_len_index(seq));
     val.push_back((int32_t)new_len);
-    return push_updates(c, idx, val, static_cast<cudaStream_t>(stream));
+    if (int rc = push_updates(c, idx, val, static_cast<cudaStream_t>(stream))) return rc;
+    return push_free_stack(c, static_cast<cudaStream_t>(stream));
 }
 
 int kv_seq_free(kv_cache* c, int32_t seq, void* stream)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_seq_free: null cache");
+    if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     std::vector<int32_t> idx, val;
     auto& pg = c->pages[seq];
@@ -436,12 +495,14 @@ int kv_seq_free(kv_cache* c, int32_t seq, void* stream)
     c->step_active = false;
     idx.push_back(c->seq_len_index(seq));
     val.push_back(0);
-    return push_updates(c, idx, val, static_cast<cudaStream_t>(stream));
+    if (int rc = push_updates(c, idx, val, static_cast<cudaStream_t>(stream))) return rc;
+    return push_free_stack(c, static_cast<cudaStream_t>(stream));
 }
 
 int kv_seq_info(kv_cache* c, int32_t seq, int32_t* len, int32_t* page_ids, int32_t capacity, int32_t* n_pages)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_seq_info: null cache");
+    if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     const auto& pg = c->pages[seq];
     if (len) *len = c->lens[seq];
@@ -456,6 +517,7 @@ static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq,
 {
     if (!c) return fail(KVC_ERR_INVALID, std::string(what) + ": null cache");
     if (int rc = check_device(c, what)) return rc;
+    if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     if (layer < 0 || layer >= c->cfg.num_layers) return fail(KVC_ERR_INVALID, std::string(what) + ": bad layer");
     if (first < 0 || n < 0 || (int64_t)first + n > c->lens[seq])
@@ -497,6 +559,7 @@ int kv_read_tokens(kv_cache* c, int32_t layer, int32_t seq, int32_t first_pos, i
 int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stream)
 {
     if (!c || !seq_ids) return fail(KVC_ERR_INVALID, "kv_begin_step: null argument");
+    if (int rc = sync_from_device(c)) return rc;
     if (batch < 1 || batch > c->cfg.max_seqs) return fail(KVC_ERR_INVALID, "kv_begin_step: batch outside 1 .. max_seqs");
     if (++c->stamp_gen == 0) {
         std::fill(c->stamp.begin(), c->stamp.end(), 0u);
@@ -581,11 +644,14 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
             KVD_CUDA(launch_step(patch, pa, st));
             ++c->launches;
         }
-        KVD_CUDA(launch_gather_pages(c->plan, (int32_t)entries, c->page_table(), c->cfg.max_pages_per_seq,
+        KVD_CUDA(launch_gather_pages(c->plan, (int32_t)entries, nullptr, c->page_table(), c->cfg.max_pages_per_seq,
                                      c->item_pages, stride, c->num_sms, st));
         ++c->launches;
     }
+    if (!c->host_only)
+        if (int rc = push_free_stack(c, static_cast<cudaStream_t>(stream))) return rc;
     c->step_active = true;
+    c->step_dev = false;
     c->step_split = split;
     c->page_stride = stride;
     c->step_batch = batch;
@@ -649,6 +715,7 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.rows = c->rows;
     p.item_pages = c->item_pages;
     p.page_stride = c->page_stride;
+    p.n_entries_dev = c->step_dev ? c->d_small + 1 : nullptr;
     p.batch = batch;
     // A fused launch may start while the previous one drains, so consecutive
     // fused launches use different work counters.
@@ -691,6 +758,81 @@ int decode_attention_append(kv_cache* c, int32_t layer, int32_t batch, const voi
 {
     if (!k_new) return fail(KVC_ERR_INVALID, "decode_attention_append: k_new must be non-null");
     return launch_attention(c, "decode_attention_append", layer, batch, q, k_new, v_new, out, softmax_scale, stream);
+}
+
+int kv_cache_device_steps(kv_cache* c, int32_t max_batch, int32_t enable, void* stream)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_cache_device_steps: null cache");
+    if (int rc = check_device(c, "kv_cache_device_steps")) return rc;
+    if (int rc = sync_from_device(c)) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    c->step_active = false;
+    if (!enable) {
+        c->dev_mode = false;
+        return KVC_OK;
+    }
+    if (max_batch < 1 || max_batch > c->cfg.max_seqs)
+        return fail(KVC_ERR_INVALID, "kv_cache_device_steps: max_batch outside 1 .. max_seqs");
+    // Work-item size from the pages now held (steps add a token per sequence).
+    const int32_t T = c->split_override
+                          ? c->split_override
+                          : auto_item_pages(c, c->pages_in_use * (int64_t)c->cfg.num_kv_heads);
+    const int32_t entries = max_batch * kMaxChunks;
+    const int32_t stride = std::max(T, (c->cfg.max_pages_per_seq + kMaxChunks - 1) / kMaxChunks) + 1;
+    if (int rc = grow_scratch(c, entries, (int64_t)entries * c->cfg.num_kv_heads, (int64_t)entries * stride, st))
+        return rc;
+    if (!c->d_free) KVD_CUDA(cudaMalloc((void**)&c->d_free, (size_t)c->cfg.num_pages * sizeof(int32_t)));
+    if (!c->d_small) KVD_CUDA(cudaMalloc((void**)&c->d_small, 2 * sizeof(int32_t)));
+    c->dev_mode = true;
+    c->dev_max_batch = max_batch;
+    c->dev_item_pages = T;
+    c->dev_entries_cap = entries;
+    c->dev_stride = stride;
+    return push_free_stack(c, st);
+}
+
+int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stream)
+{
+    if (!c || !seq_ids) return fail(KVC_ERR_INVALID, "kv_begin_step_device: null argument");
+    if (!c->dev_mode) return fail(KVC_ERR_INVALID, "kv_begin_step_device: device steps are not enabled");
+    if (batch < 1 || batch > c->dev_max_batch)
+        return fail(KVC_ERR_INVALID, "kv_begin_step_device: batch outside 1 .. max_batch");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    StepDevArgs a;
+    a.batch = batch;
+    a.item_pages = c->dev_item_pages;
+    a.max_pages = c->cfg.max_pages_per_seq;
+    a.max_entries = c->dev_entries_cap;
+    a.seq_ids = seq_ids;
+    a.free_pages = c->d_free;
+    a.free_top = c->d_small;
+    a.step_seq = c->step_seq;
+    a.seq_len = c->seq_len_dev();
+    a.page_table = c->page_table();
+    a.plan = c->plan;
+    a.rows = c->rows;
+    a.n_entries = c->d_small + 1;
+    a.err = c->err;
+    KVD_CUDA(launch_step_device(a, st));
+    ++c->launches;
+    KVD_CUDA(launch_gather_pages(c->plan, c->dev_entries_cap, c->d_small + 1, c->page_table(),
+                                 c->cfg.max_pages_per_seq, c->item_pages, c->dev_stride, c->num_sms, st));
+    ++c->launches;
+    c->dev_dirty = true;
+    c->step_active = true;
+    c->step_dev = true;
+    c->step_split = true;   // the row split is only known on the device: always run the merge pass
+    c->step_batch = batch;
+    c->step_entries = c->dev_entries_cap;
+    c->page_stride = c->dev_stride;
+    return KVC_OK;
+}
+
+int kv_cache_sync(kv_cache* c)
+{
+    if (!c) return fail(KVC_ERR_INVALID, "kv_cache_sync: null cache");
+    if (c->host_only) return KVC_OK;
+    return sync_from_device(c);
 }
 
 int kv_selftest_wait_timeout(int64_t limit_ns, int32_t* status, void* stream)

@@ -71,6 +71,24 @@ struct PlanArgs {
     int32_t* err;
 };
 
+// kv_begin_step_device: the step's lazy allocation and plan, on the device.
+struct StepDevArgs {
+    int32_t batch;
+    int32_t item_pages;       // target pages per work item (T)
+    int32_t max_pages;        // page-table row length
+    int32_t max_entries;      // capacity of plan
+    const int32_t* seq_ids;   // [batch] sequence ids (device)
+    int32_t* free_pages;      // device free stack; the next page is free_pages[*free_top - 1]
+    int32_t* free_top;
+    int32_t* step_seq;
+    int32_t* seq_len;
+    int32_t* page_table;
+    PlanEntry* plan;
+    int2* rows;
+    int32_t* n_entries;       // out: plan entries of the step
+    int32_t* err;
+};
+
 struct ScatterI32 {
     int32_t n;
     int32_t idx[kScatterMax];
@@ -113,6 +131,7 @@ struct DecodeParams {
     const int2* rows;         // [batch]: (first partial slot, items) per batch row
     const int32_t* item_pages;// [entries][page_stride]: page ids of each plan entry's pages
     int32_t page_stride;
+    const int32_t* n_entries_dev; // device-built plan: entries live here (n_items is then a bound)
     int32_t batch;
     uint32_t* queue;          // [0] next item, [1] warps finished
     int32_t* err;
@@ -149,8 +168,11 @@ cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, cudaStream
 cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
 // Copy each plan entry's page ids from the page table into item_pages
 // ([entries][stride]), so the decode kernel reads them alongside the entry.
-cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* page_table,
-                                int32_t max_pages, int32_t* item_pages, int32_t stride, int num_sms, cudaStream_t st);
+// entries_dev (if non-null) holds the entry count; `entries` is then its bound.
+cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const int32_t* entries_dev,
+                                const int32_t* page_table, int32_t max_pages, int32_t* item_pages, int32_t stride,
+                                int num_sms, cudaStream_t st);
+cudaError_t launch_step_device(const StepDevArgs& a, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
 cudaError_t launch_wait_timeout_check(uint64_t limit_ns, int32_t* status, cudaStream_t st);
 

@@ -237,7 +237,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     noalloc_plan_kernel<<<1, 1024, 0, st>>>(pa);
     if (cudaError_t e = cudaGetLastError(); e != cudaSuccess) return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     int32_t* item_pages = reinterpret_cast<int32_t*>(scratch + off_pages);
-    if (cudaError_t e = launch_gather_pages(pa.plan, (int32_t)entries, page_table, max_pages, item_pages, stride,
+    if (cudaError_t e = launch_gather_pages(pa.plan, (int32_t)entries, nullptr, page_table, max_pages, item_pages, stride,
                                             num_sms, st);
         e != cudaSuccess)
         return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
@@ -253,6 +253,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.rows = pa.rows;
     p.item_pages = item_pages;
     p.page_stride = stride;
+    p.n_entries_dev = nullptr;
     p.batch = batch;
     p.queue = pa.queue;
     p.err = pa.err;

@@ -26,6 +26,7 @@ KVC_FLAG_HOST_ONLY = 1
 KVC_DEVERR_PAGE_RANGE = 1
 KVC_DEVERR_WAIT_TIMEOUT = 2
 KVC_DEVERR_SEQ_RANGE = 4
+KVC_DEVERR_OOM = 8
 
 _NAMES = {KVC_ERR_INVALID: "INVALID", KVC_ERR_OOM: "OOM", KVC_ERR_CUDA: "CUDA",
           KVC_ERR_PAGE_TABLE: "PAGE_TABLE", KVC_ERR_UNSUPPORTED: "UNSUPPORTED",
@@ -75,6 +76,9 @@ _SIGS = {
     "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
     "decode_attention_append": [_P, _I32, _I32, _P, _P, _P, _P, ctypes.c_float, _P],
     "kv_selftest_wait_timeout": [_I64, _P, _P],
+    "kv_cache_device_steps": [_P, _I32, _I32, _P],
+    "kv_begin_step_device": [_P, _I32, _P, _P],
+    "kv_cache_sync": [_P],
     "decode_attention_noalloc": [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _I32, _P, _P, _P,
                                  ctypes.c_float, _P, _P],
 }
@@ -145,7 +149,8 @@ def kv_cache_set_page_order(h, order):
 def kv_cache_query(h, raise_on_device_error: bool = True) -> kvc_stats:
     s = kvc_stats()
     rc = load().kv_cache_query(h, ctypes.byref(s))
-    if rc != KVC_OK and (raise_on_device_error or rc not in (KVC_ERR_PAGE_TABLE, KVC_ERR_DEVICE)):
+    # A status caused by a device-side error flag still fills the stats.
+    if rc != KVC_OK and (raise_on_device_error or s.device_error == 0):
         _check(rc, "kv_cache_query")
     return s
 
@@ -225,6 +230,18 @@ def decode_attention_noalloc(k_pool, v_pool, num_pages: int, num_q_heads: int, n
                                            ctypes.addressof(arr), _ptr(q), _ptr(out), float(softmax_scale),
                                            _ptr(device_error), _stream(stream)),
            "decode_attention_noalloc")
+
+
+def kv_cache_device_steps(h, max_batch: int, enable: bool = True, stream=None):
+    _check(load().kv_cache_device_steps(h, max_batch, 1 if enable else 0, _stream(stream)), "kv_cache_device_steps")
+
+
+def kv_begin_step_device(h, batch: int, seq_ids_dev, stream=None):
+    _check(load().kv_begin_step_device(h, batch, _ptr(seq_ids_dev), _stream(stream)), "kv_begin_step_device")
+
+
+def kv_cache_sync(h):
+    _check(load().kv_cache_sync(h), "kv_cache_sync")
 
 
 def kv_selftest_wait_timeout(limit_ns: int, status, stream=None):

@@ -1,0 +1,138 @@
+"""Device-side decode steps (kv_begin_step_device) and a whole decode step
+captured once into a CUDA graph and replayed: same pages, same lengths and
+bit-identical outputs as host-driven steps; exhaustion is reported."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import PagePoolModel
+from paper_2603_12707_gb300 import kvdecode as kd
+from paper_2603_12707_gb300 import workloads as wl
+
+from _gpu_common import Tracked, assert_close, bf16_to_f64
+
+pytestmark = pytest.mark.gpu
+
+SPLIT = 3   # same work-item size for both sides, so outputs are bit-identical
+
+
+def _pair(cfg, extra=24):
+    a = Tracked(cfg, extra_tokens=extra, split_pages=SPLIT, keep_host=True)
+    b = Tracked(cfg, extra_tokens=extra, split_pages=SPLIT, keep_host=False)
+    return a, b
+
+
+@pytest.mark.parametrize("Hq,Hkv,d,lens", [
+    (8, 8, 128, [0, 15, 16, 31, 200, 47]),
+    (28, 4, 128, [1, 16, 300, 2100]),
+])
+def test_device_steps_match_host_steps(kvlib, Hq, Hkv, d, lens):
+    cfg = wl.custom("devstep", 2, Hq, Hkv, d, len(lens), lens=lens, seed=5 + Hq, page_order="shuffled")
+    a, b = _pair(cfg)
+    kd.kv_cache_device_steps(b.sess.h, cfg.batch)
+    ids = torch.tensor(b.sess.seq_ids, dtype=torch.int32, device="cuda")
+    for step in range(20):
+        a.begin_step()
+        kd.kv_begin_step_device(b.sess.h, cfg.batch, ids)
+        b.step += 1
+        b.sess.lens += 1
+        for layer in range(cfg.num_layers):
+            oa, q, _, _ = a.run_layer(layer, fused=True)
+            ob, _, _, _ = b.run_layer(layer, fused=(layer % 2 == 0))
+            torch.cuda.synchronize()
+            assert torch.equal(oa, ob), (step, layer)
+            if step in (0, 19):
+                ref, vmax = a.oracle(layer, q)
+                assert_close(bf16_to_f64(ob), ref, vmax, gqa=Hq > Hkv)
+    # the host view after a sync: same lengths and pages as host steps
+    kd.kv_cache_sync(b.sess.h)
+    for sa, sb in zip(a.sess.seq_ids, b.sess.seq_ids):
+        assert kd.kv_seq_info(a.sess.h, sa) == kd.kv_seq_info(b.sess.h, sb)
+    st_a, st_b = kd.kv_cache_query(a.sess.h), kd.kv_cache_query(b.sess.h)
+    assert (st_a.pages_in_use, st_a.free_pages) == (st_b.pages_in_use, st_b.free_pages)
+    # host calls keep working after device steps (allocator state came back)
+    b.begin_step()
+    a.begin_step()
+    for sa, sb in zip(a.sess.seq_ids, b.sess.seq_ids):
+        assert kd.kv_seq_info(a.sess.h, sa) == kd.kv_seq_info(b.sess.h, sb)
+    a.close()
+    b.close()
+
+
+def test_captured_step_replays_like_host_steps(kvlib):
+    cfg = wl.custom("graph", 4, 28, 4, 128, 5, lens=[100, 16, 999, 35, 512], seed=61, page_order="shuffled")
+    a, b = _pair(cfg, extra=40)
+    L = cfg.num_layers
+    ins = [wl.step_inputs(cfg, 0, l, "cuda") for l in range(L)]
+    outs = [torch.empty_like(i[0]) for i in ins]
+    ids = torch.tensor(b.sess.seq_ids, dtype=torch.int32, device="cuda")
+    kd.kv_cache_device_steps(b.sess.h, cfg.batch)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        # one eager step first so no lazy initialisation happens inside the capture
+        kd.kv_begin_step_device(b.sess.h, cfg.batch, ids, s)
+        for l in range(L):
+            kd.decode_attention_append(b.sess.h, l, cfg.batch, ins[l][0], ins[l][1], ins[l][2], outs[l], 0.0, s)
+    s.synchronize()
+    a.sess.begin_step()
+    for l in range(L):
+        oa = torch.empty_like(outs[l])
+        a.sess.append_attend(l, ins[l][0], ins[l][1], ins[l][2], oa)
+        torch.cuda.synchronize()
+        assert torch.equal(oa, outs[l])
+    with torch.cuda.graph(g, stream=s):
+        cs = torch.cuda.current_stream()
+        kd.kv_begin_step_device(b.sess.h, cfg.batch, ids, cs)
+        for l in range(L):
+            kd.decode_attention_append(b.sess.h, l, cfg.batch, ins[l][0], ins[l][1], ins[l][2], outs[l], 0.0, cs)
+    for rep in range(12):
+        g.replay()
+        a.sess.begin_step()
+        refs = []
+        for l in range(L):
+            oa = torch.empty_like(outs[l])
+            a.sess.append_attend(l, ins[l][0], ins[l][1], ins[l][2], oa)
+            refs.append(oa)
+        torch.cuda.synchronize()
+        for l in range(L):
+            assert torch.equal(refs[l], outs[l]), (rep, l)
+    kd.kv_cache_sync(b.sess.h)
+    for sa, sb in zip(a.sess.seq_ids, b.sess.seq_ids):
+        assert kd.kv_seq_info(a.sess.h, sa) == kd.kv_seq_info(b.sess.h, sb)
+    a.close()
+    b.close()
+
+
+def test_device_step_reports_an_exhausted_pool(kvlib):
+    """5 pages, 3 sequences of 16 tokens (3 pages held): the next step needs a
+    page for each; the first two rows (batch order) get them, the third is
+    left at its length and the pool exhaustion is reported."""
+    cfg = kd.make_config(1, 8, 8, 64, 5, 4, 8)
+    h = kd.kv_cache_create(cfg)
+    seqs = [kd.kv_seq_create(h) for _ in range(3)]
+    for s_ in seqs:
+        kd.kv_seq_reserve(h, s_, 16)
+    kd.kv_cache_device_steps(h, 3)
+    ids = torch.tensor(seqs, dtype=torch.int32, device="cuda")
+    kd.kv_begin_step_device(h, 3, ids)
+    torch.cuda.synchronize()
+    with pytest.raises(kd.KVDecodeError) as ei:
+        kd.kv_cache_query(h)
+    assert ei.value.code == kd.KVC_ERR_OOM
+    st = kd.kv_cache_query(h, raise_on_device_error=False)
+    assert st.device_error & kd.KVC_DEVERR_OOM
+    assert st.free_pages == 0 and st.pages_in_use == 5
+    assert [kd.kv_seq_info(h, s_)[0] for s_ in seqs] == [17, 17, 16]
+    # the host allocator model agrees on which pages went where
+    m = PagePoolModel(5, 16, 4, 8)
+    for _ in range(3):
+        m.seq_create()
+    for i in range(3):
+        m.seq_reserve(i, 16)
+    m.seq_reserve(0, 1)
+    m.seq_reserve(1, 1)
+    for i, s_ in enumerate(seqs):
+        assert kd.kv_seq_info(h, s_)[1] == m.pages[i]
+    kd.kv_cache_destroy(h)
