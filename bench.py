@@ -192,7 +192,7 @@ def run_gpu(args, rank, world):
         import dataclasses
         cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
     stream = torch.cuda.Stream()
-    total_steps = args.warmup + args.steps + (args.steps if not args.no_e2e else 0) + 1
+    total_steps = args.warmup + args.steps + (args.steps if not args.no_e2e else 0) + 2
     t_setup = time.perf_counter()
     with torch.cuda.stream(stream):
         sess = DecodeSession(cfg, extra_tokens=total_steps + 1, device="cuda", stream=stream,
@@ -208,12 +208,46 @@ def run_gpu(args, rank, world):
     log(f"[rank {rank}] setup {time.perf_counter() - t_setup:.1f} s; pool "
         f"{sess.query().pool_bytes / 2**30:.1f} GiB")
 
+    graphs = None
+    if args.graph:
+        # The whole step as two CUDA graphs: the device-side kv_begin_step
+        # (page pops, lengths, split plan) and the L fused layers.  Replays
+        # need no host work; an event between the two times the layers.
+        ids_dev = torch.tensor(sess.seq_ids, dtype=torch.int32, device="cuda")
+        kd.kv_cache_device_steps(sess.h, B, True, stream)
+
+        def layers():
+            for l in range(L):
+                sess.append_attend(l, qs[l], ks[l], vs[l], outs[l])
+
+        with torch.cuda.stream(stream):
+            kd.kv_begin_step_device(sess.h, B, ids_dev, stream)   # eager step: nothing lazy in the capture
+            layers()
+        sess.lens += 1
+        stream.synchronize()
+        n0 = sess.query().kernel_launches
+        g_begin, g_layers = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_begin, stream=stream):
+            kd.kv_begin_step_device(sess.h, B, ids_dev, stream)
+        with torch.cuda.graph(g_layers, stream=stream):
+            layers()
+        graphs = (g_begin, g_layers, sess.query().kernel_launches - n0)
+
     def step(events=None):
         """One decode step.  events: per-step event list to time the attention
         launches.  Unfused: a pair around every decode_attention.  Fused: one
         event after kv_begin_step and one after the last layer (the fused
         launches are PDL-chained, and an event between two of them would cut
         the overlap), so a launch's time is the span over L."""
+        if graphs is not None:
+            graphs[0].replay()
+            if events is not None:
+                events[0].record(stream)
+            graphs[1].replay()
+            if events is not None:
+                events[1].record(stream)
+            sess.lens += 1
+            return
         sess.begin_step()
         if events is not None and not args.unfused:
             events[0].record(stream)
@@ -268,7 +302,10 @@ def run_gpu(args, rank, world):
         attn_bytes.append(a if args.unfused else a + p)   # the fused kernel also writes the new K/V
     st = sess.query()
     assert st.device_error == 0, st.device_error
-    timed_launches = st.kernel_launches - launches0
+    # graph replays do not pass through the library: count the captured launches
+    timed_launches = graphs[2] * args.steps if graphs is not None else st.kernel_launches - launches0
+    if graphs is not None:
+        kd.kv_cache_device_steps(sess.h, B, False, stream)   # host-driven steps from here on
 
     # ---- end to end: host inputs -> device -> host outputs, every step
     e2e = None
@@ -342,9 +379,13 @@ def main():
                     help="target pages per work item (0: the library's automatic choice)")
     ap.add_argument("--unfused", action="store_true",
                     help="kv_append and decode_attention as two launches per layer (default: one fused launch)")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay each step from CUDA graphs (device-side kv_begin_step, fused layers)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     args = ap.parse_args()
+    if args.graph and args.unfused:
+        ap.error("--graph captures the fused layers; drop --unfused")
     if args.warmup < 3:
         log("warning: fewer than 3 warm-up steps")
 
@@ -406,6 +447,7 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {**describe(cfg), "l2": "each step streams the whole cache (far larger than the 129 MB L2)",
                    "split_pages": args.split_pages or "auto",
+                   "step_driver": "cuda_graph" if args.graph else "host",
                    "parallelism": f"replicas x{world}"},
         "steps_per_s": round(steps_per_s * 1.0, 3),
         "pct_of_measured_hbm": round(100 * gbs / world / peak, 2),
@@ -417,8 +459,8 @@ def main():
                      "algorithmic_bytes_per_launch": int(attn_bytes), "avg_launch_ms": round(attn_ms, 4)},
         "clocks": r["clocks"],
         "gpu_launches": r["launches"],
-        "step_kernels": "kv_begin_step + per layer " + ("kv_append, decode_attention" if args.unfused
-                                                          else "decode_attention_append (fused, PDL)"),
+        "step_kernels": ("kv_begin_step" + ("_device (CUDA-graph replay)" if args.graph else "") + " + per layer "
+                         + ("kv_append, decode_attention" if args.unfused else "decode_attention_append (fused, PDL)")),
     }
     if r["e2e"]:
         e = r["e2e"]

@@ -92,7 +92,8 @@ __global__ void __launch_bounds__(1024)
 // The same step on the device (graph-replayable, no host input): rows in
 // batch order reserve position len; a row whose position opens a page takes
 // the next page of the device free stack, in batch order (the same pages the
-// host allocator would hand out); then the split plan, rows in batch order.
+// host allocator would hand out); then the split plan, rows longest first
+// (stable, as on the host) when the batch fits one block, else in batch order.
 __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
 {
     __shared__ int s_top;
@@ -134,11 +135,36 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
     }
     __syncthreads();
     if (threadIdx.x == 0) *a.free_top = top0 - min(carry, top0);
+
+    // Row order: the rank of row b counts the rows with more pages, and the
+    // rows with as many pages that come before b.
+    __shared__ int s_np[1024];
+    __shared__ int s_order[1024];
+    const bool ordered = a.batch <= (int)blockDim.x;
+    if (ordered) {
+        const int b = threadIdx.x;
+        int np = 0;
+        if (b < a.batch) {
+            np = (max(1, a.seq_len[a.step_seq[b]]) + kPageSize - 1) / kPageSize;
+            s_np[b] = np;
+        }
+        __syncthreads();
+        if (b < a.batch) {
+            int rank = 0;
+            for (int j = 0; j < a.batch; ++j) {
+                const int o = s_np[j];
+                rank += (o > np || (o == np && j < b)) ? 1 : 0;
+            }
+            s_order[rank] = b;
+        }
+        __syncthreads();
+    }
     carry = 0;
     for (int base = 0; base < a.batch; base += blockDim.x) {
-        const int b = base + threadIdx.x;
+        const int i = base + threadIdx.x;
+        const int b = (ordered && i < a.batch) ? s_order[i] : i;
         int seq = 0, len = 0, np = 0, nch = 0;
-        if (b < a.batch) {
+        if (i < a.batch) {
             seq = a.step_seq[b];
             len = max(1, a.seq_len[seq]);
             np = (len + kPageSize - 1) / kPageSize;
@@ -155,7 +181,7 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
             chunk_range(np, nch, c, &first, &n);
             a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
         }
-        if (b < a.batch) a.rows[b] = make_int2(off, nch);
+        if (i < a.batch) a.rows[b] = make_int2(off, nch);
         carry += total;
     }
     if (threadIdx.x == 0) *a.n_entries = min(carry, a.max_entries);
