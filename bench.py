@@ -358,6 +358,90 @@ def run_gpu(args, rank, world):
             "clocks": clocks.summary(), "e2e": e2e, "cfg": cfg, "L": L}
 
 
+def run_varlen_write(args, rank, world):
+    """Time kv_write_varlen: the workload's whole batch of cached prefixes
+    (vision tokens + prompt + generated), packed, written into every layer
+    pool in one call per step.  Bytes = packed K/V read + pool pages written."""
+    import torch
+    from paper_2603_12707_gb300 import _build, kvdecode as kd, workloads as wl
+    from paper_2603_12707_gb300.harness import DecodeSession
+
+    dev = int(os.environ.get("LOCAL_RANK", 0))
+    torch.cuda.set_device(dev)
+    if rank == 0:
+        _build.build_library()
+    if world > 1:
+        torch.distributed.barrier()
+    cfg = wl.CONFIGS[args.config]
+    if args.phys_layers:
+        import dataclasses
+        cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
+    stream = torch.cuda.Stream()
+    sess = DecodeSession(cfg, extra_tokens=1, device="cuda", stream=stream)
+    lens = [int(n) for n in sess.lens0]
+    L = cfg.phys_layers
+    src_bytes = 2 * sum(lens) * cfg.num_kv_heads * cfg.head_dim * 2 * L
+    if src_bytes > 64 * 2**30:
+        raise SystemExit(f"packed source of {src_bytes / 2**30:.0f} GiB: pass --phys-layers")
+    k, v, cu = wl.packed_prefix(cfg, range(L), lens, "cuda")
+    torch.cuda.synchronize()
+
+    def step():
+        kd.kv_write_varlen(sess.h, 0, L, sess.seq_ids, cu, k, v, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    n0 = sess.query().kernel_launches
+    with ClockSampler(gpu_smi_id(torch, dev)) as clocks:
+        for a, b in ev:
+            a.record(stream)
+            step()
+            b.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    st = sess.query()
+    assert st.device_error == 0
+    launches = st.kernel_launches - n0
+    ms = sum(a.elapsed_time(b) for a, b in ev)
+    sess.close()
+    return {"ms": ms, "bytes": 2 * src_bytes, "launches": launches, "clocks": clocks.summary(), "cfg": cfg,
+            "blocks": len(lens), "rows": cu[-1]}
+
+
+def varlen_main(args, rank, world):
+    import torch
+    r = run_varlen_write(args, rank, world)
+    ms = reduce_max(torch, r["ms"], world)
+    gbs = r["bytes"] * args.steps * world / (ms / 1e3) / 1e9
+    peak, peak_kind = measured_peaks()
+    cfg = r["cfg"]
+    out = {
+        "metric": "paged varlen K/V bulk write (prefix handoff), HBM GB/s read + write", "value": round(gbs, 2),
+        "unit": "GB/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {**describe(cfg), "blocks": r["blocks"], "packed_rows": r["rows"],
+                   "l2": "each step reads and writes the whole prefix batch (far larger than the 129 MB L2)"
+                         if r["bytes"] > 2**30 else "fits in L2: launch-bound, not a roofline number",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "kernel": "kv_write_varlen", "achieved": round(gbs / world, 2), "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": round(gbs / world / peak, 4), "traffic": None,
+                     "algorithmic_bytes_per_launch": int(r["bytes"] / max(1, r["launches"] // args.steps)),
+                     "avg_launch_ms": round(ms / max(1, r["launches"]), 4)},
+        "clocks": r["clocks"], "gpu_launches": r["launches"],
+    }
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out))
+
+
 def reduce_max(torch, x, world):
     if world == 1:
         return x
@@ -381,6 +465,8 @@ def main():
                     help="kv_append and decode_attention as two launches per layer (default: one fused launch)")
     ap.add_argument("--graph", action="store_true",
                     help="replay each step from CUDA graphs (device-side kv_begin_step, fused layers)")
+    ap.add_argument("--varlen-write", action="store_true",
+                    help="time the packed varlen bulk K/V write of the workload's prefixes instead of decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     args = ap.parse_args()
@@ -430,6 +516,9 @@ def main():
     import torch
     if world > 1:
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0))))
+    if args.varlen_write:
+        varlen_main(args, rank, world)
+        return
     r = run_gpu(args, rank, world)
     cfg, L = r["cfg"], r["L"]
     ms = reduce_max(torch, r["ms"], world)

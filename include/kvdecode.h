@@ -162,6 +162,28 @@ KVC_API int kv_seq_info(kv_cache *cache, int32_t seq_id, int32_t *len, int32_t *
 KVC_API int kv_write_tokens(kv_cache *cache, int32_t layer, int32_t seq_id, int32_t first_pos,
                     int32_t n, const void *k, const void *v, void *stream);
 
+/* Bulk write of a packed variable-length batch of token blocks, in one launch
+ * (one per 512 non-empty blocks): the vision-prefix K/V handed over at the
+ * modality boundary plus the prompt, for many sequences and layers at once
+ * (Sec. 5.1 handoff; Sec. 5.4 "Flash Attention Varlen for Packed Prefill":
+ * one packed tensor with cumulative lengths, one launch instead of one per
+ * sequence).  Block i holds the rows cu_seqlens[i] ..
+ * cu_seqlens[i+1]-1 of k and v and goes to positions first_pos[i] ..
+ * first_pos[i] + n_i - 1 of sequence seq_ids[i], in layers layer_first ..
+ * layer_first + n_layers - 1.
+ *   seq_ids, first_pos, cu_seqlens: host arrays of n_blocks, n_blocks and
+ *     n_blocks + 1 entries; cu_seqlens[0] == 0 and non-decreasing; first_pos
+ *     NULL means 0 for every block.  Blocks may name the same sequence but
+ *     not the same position (KVC_ERR_INVALID); empty blocks are skipped.
+ *   k, v: device, [n_layers][cu_seqlens[n_blocks]][H_kv][d_h] bf16, 16-byte
+ *     aligned, read when the kernel runs.
+ * The positions must already be reserved (kv_seq_reserve on this stream or
+ * before it).  A page id outside the pool found by the kernel sets
+ * KVC_DEVERR_PAGE_RANGE and that page is not written. */
+KVC_API int kv_write_varlen(kv_cache *cache, int32_t layer_first, int32_t n_layers, int32_t n_blocks,
+                    const int32_t *seq_ids, const int32_t *first_pos, const int32_t *cu_seqlens,
+                    const void *k, const void *v, void *stream);
+
 /* Copy positions [first_pos, first_pos + n) of one layer back into logical
  * order: k_out, v_out device [n][H_kv][d_h] bf16. */
 KVC_API int kv_read_tokens(kv_cache *cache, int32_t layer, int32_t seq_id, int32_t first_pos,

@@ -216,6 +216,71 @@ __global__ void token_copy_kernel(const TokenCopyArgs a)
     }
 }
 
+// Bulk write of packed token blocks.  CTA x finds its block by a binary
+// search over tile_start, reads the tile's page id once, then its threads
+// stream the tile in the page's order ([H_kv][slot][D], 16-byte chunks, four
+// per thread in flight) with streaming loads and stores: the source is read
+// once and the pages are not read back soon.
+constexpr int kVarlenThreads = 256;
+constexpr int kVarlenUnroll = 4;
+
+__global__ void __launch_bounds__(kVarlenThreads) varlen_write_kernel(const __grid_constant__ VarlenWriteArgs a)
+{
+    const int tile = blockIdx.x;
+    int lo = 0, hi = a.n_blocks - 1;   // the last block with tile_start <= tile
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (a.tile_start[mid] <= tile) lo = mid;
+        else hi = mid - 1;
+    }
+    const int first = a.first_pos[lo];
+    const int page_idx = first / kPageSize + (tile - a.tile_start[lo]);
+    const int p0 = max(first, page_idx * kPageSize);
+    const int p1 = min(first + a.n_tok[lo], (page_idx + 1) * kPageSize);
+    const int nt = p1 - p0;
+    const int32_t pid = a.page_table[(int64_t)a.seq[lo] * a.max_pages + page_idx];
+    if (pid < 0 || pid >= a.num_pages) {
+        if (threadIdx.x == 0) flag_error(a.err, 1);
+        return;
+    }
+    const int cpr = a.D / 8;   // 16-byte chunks per (token, head) row
+    const int total = a.H_kv * nt * cpr;
+    const int64_t layer = blockIdx.y;
+    const uint4* sk = reinterpret_cast<const uint4*>(a.k + layer * a.src_layer_stride);
+    const uint4* sv = reinterpret_cast<const uint4*>(a.v + layer * a.src_layer_stride);
+    uint4* dk = reinterpret_cast<uint4*>(a.pool_k + layer * a.pool_layer_stride) +
+                (int64_t)pid * a.H_kv * kPageSize * cpr;
+    uint4* dv = reinterpret_cast<uint4*>(a.pool_v + layer * a.pool_layer_stride) +
+                (int64_t)pid * a.H_kv * kPageSize * cpr;
+    const int64_t tok0 = (int64_t)a.src_row[lo] + (p0 - first);
+    const int slot0 = p0 - page_idx * kPageSize;
+    for (int base = threadIdx.x; base < total; base += kVarlenUnroll * kVarlenThreads) {
+        uint4 rk[kVarlenUnroll], rv[kVarlenUnroll];
+        int64_t doff[kVarlenUnroll];
+#pragma unroll
+        for (int u = 0; u < kVarlenUnroll; ++u) {
+            const int idx = base + u * kVarlenThreads;
+            if (idx < total) {
+                const int c = idx % cpr;
+                const int r = idx / cpr;
+                const int h = r / nt;
+                const int t = r - h * nt;
+                const int64_t soff = ((tok0 + t) * a.H_kv + h) * cpr + c;
+                doff[u] = ((int64_t)h * kPageSize + slot0 + t) * cpr + c;
+                rk[u] = __ldcs(sk + soff);
+                rv[u] = __ldcs(sv + soff);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kVarlenUnroll; ++u) {
+            if (base + u * kVarlenThreads < total) {
+                __stcs(dk + doff[u], rk[u]);
+                __stcs(dv + doff[u], rv[u]);
+            }
+        }
+    }
+}
+
 // kv_append: one thread per 16-byte chunk of k_new / v_new ([B][H_kv][D]);
 // the chunk goes to slot (len-1) % P of page page_table[seq][(len-1) / P].
 __global__ void append_kernel(const AppendArgs a)
@@ -324,6 +389,13 @@ cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st)
     int64_t blocks = (total + 255) / 256;
     if (blocks > 65535) blocks = 65535;
     token_copy_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_varlen_write(const VarlenWriteArgs& a, int n_layers, cudaStream_t st)
+{
+    if (a.n_tiles <= 0 || n_layers <= 0) return cudaSuccess;
+    varlen_write_kernel<<<dim3((unsigned)a.n_tiles, (unsigned)n_layers), kVarlenThreads, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -556,6 +556,88 @@ int kv_read_tokens(kv_cache* c, int32_t layer, int32_t seq, int32_t first_pos, i
     return token_copy(c, "kv_read_tokens", layer, seq, first_pos, n, k_out, v_out, 0, stream);
 }
 
+int kv_write_varlen(kv_cache* c, int32_t layer_first, int32_t n_layers, int32_t n_blocks, const int32_t* seq_ids,
+                    const int32_t* first_pos, const int32_t* cu_seqlens, const void* k, const void* v, void* stream)
+{
+    if (!c || (n_blocks > 0 && (!seq_ids || !cu_seqlens)))
+        return fail(KVC_ERR_INVALID, "kv_write_varlen: null argument");
+    if (int rc = sync_from_device(c)) return rc;
+    if (n_layers < 1 || n_layers > 65535 || layer_first < 0 || (int64_t)layer_first + n_layers > c->cfg.num_layers)
+        return fail(KVC_ERR_INVALID, "kv_write_varlen: layers outside the cache");
+    if (n_blocks < 0) return fail(KVC_ERR_INVALID, "kv_write_varlen: negative block count");
+    if (n_blocks == 0) return KVC_OK;
+    if (cu_seqlens[0] != 0) return fail(KVC_ERR_INVALID, "kv_write_varlen: cu_seqlens[0] must be 0");
+    std::vector<int32_t> order((size_t)n_blocks);
+    for (int32_t i = 0; i < n_blocks; ++i) {
+        if (int rc = check_seq(c, seq_ids[i])) return rc;
+        const int64_t n = (int64_t)cu_seqlens[i + 1] - cu_seqlens[i];
+        const int64_t f = first_pos ? first_pos[i] : 0;
+        if (n < 0) return fail(KVC_ERR_INVALID, "kv_write_varlen: cu_seqlens must not decrease");
+        if (f < 0 || f + n > c->lens[seq_ids[i]])
+            return fail(KVC_ERR_INVALID, "kv_write_varlen: positions outside the reserved length");
+        order[i] = i;
+    }
+    // Two blocks may not write the same position of a sequence.
+    auto fpos = [&](int32_t i) { return first_pos ? first_pos[i] : 0; };
+    std::sort(order.begin(), order.end(), [&](int32_t x, int32_t y) {
+        return seq_ids[x] != seq_ids[y] ? seq_ids[x] < seq_ids[y] : fpos(x) < fpos(y);
+    });
+    int64_t end = 0;   // end of the blocks seen so far in the current sequence
+    for (int32_t j = 0; j < n_blocks; ++j) {
+        const int32_t y = order[j];
+        const int64_t n = (int64_t)cu_seqlens[y + 1] - cu_seqlens[y];
+        if (j == 0 || seq_ids[order[j - 1]] != seq_ids[y]) end = 0;
+        if (n == 0) continue;
+        if (fpos(y) < end) return fail(KVC_ERR_INVALID, "kv_write_varlen: blocks overlap in a sequence");
+        end = fpos(y) + n;
+    }
+    const int64_t rows = cu_seqlens[n_blocks];
+    if (rows == 0) return KVC_OK;
+    if (!k || !v || !aligned16(k) || !aligned16(v))
+        return fail(KVC_ERR_INVALID, "kv_write_varlen: k / v must be non-null and 16-byte aligned");
+    if (int rc = check_device(c, "kv_write_varlen")) return rc;
+
+    VarlenWriteArgs a;
+    a.pool_k = c->k_pool(layer_first);
+    a.pool_v = c->v_pool(layer_first);
+    a.pool_layer_stride = (int64_t)c->layer_elems;
+    a.k = static_cast<const uint16_t*>(k);
+    a.v = static_cast<const uint16_t*>(v);
+    a.src_layer_stride = rows * c->cfg.num_kv_heads * c->cfg.head_dim;
+    a.page_table = c->page_table();
+    a.num_pages = c->cfg.num_pages;
+    a.max_pages = c->cfg.max_pages_per_seq;
+    a.H_kv = c->cfg.num_kv_heads;
+    a.D = c->cfg.head_dim;
+    a.err = c->err;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // Blocks go kVarlenMax at a time (empty ones skipped), one launch each.
+    auto flush = [&]() -> int {
+        if (a.n_blocks == 0) return KVC_OK;
+        a.n_tiles = a.tile_start[a.n_blocks];
+        KVD_CUDA(launch_varlen_write(a, n_layers, st));
+        ++c->launches;
+        a.n_blocks = 0;
+        return KVC_OK;
+    };
+    a.n_blocks = 0;
+    a.tile_start[0] = 0;
+    for (int32_t i = 0; i < n_blocks; ++i) {
+        const int32_t n = cu_seqlens[i + 1] - cu_seqlens[i];
+        if (n == 0) continue;
+        const int32_t f = fpos(i);
+        const int32_t j = a.n_blocks;
+        a.seq[j] = seq_ids[i];
+        a.first_pos[j] = f;
+        a.n_tok[j] = n;
+        a.src_row[j] = cu_seqlens[i];
+        a.tile_start[j + 1] = a.tile_start[j] + ((f + n - 1) / kPageSize - f / kPageSize + 1);
+        if (++a.n_blocks == kVarlenMax)
+            if (int rc = flush()) return rc;
+    }
+    return flush();
+}
+
 int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stream)
 {
     if (!c || !seq_ids) return fail(KVC_ERR_INVALID, "kv_begin_step: null argument");

@@ -14,6 +14,7 @@ constexpr int kMaxChunks = 32;         // work items per (row, KV head) at most
 constexpr int kMaxItemPages = 1024;    // largest target item size a caller may request
 constexpr int kPatchMax = 1024;        // step entries carried in one launch's parameters
 constexpr int kScatterMax = 2048;      // int32 updates carried in one launch's parameters
+constexpr int kVarlenMax = 512;        // token blocks carried in one bulk-write launch's parameters
 
 // One work item of a step's split plan: consecutive pages [first_page,
 // first_page + n_pages) of batch row b.  Items are expanded over the H_kv
@@ -108,6 +109,30 @@ struct TokenCopyArgs {
     int32_t* err;
 };
 
+// Bulk write of packed variable-length token blocks into the pools (prefill
+// or the vision-prefix handoff).  A tile is the part of one block's position
+// range that falls in one page; CTA (x, y) writes tile x of layer
+// layer_first + y.
+struct VarlenWriteArgs {
+    uint16_t* pool_k;            // pool of the first layer written, [num_pages][H_kv][P][D]
+    uint16_t* pool_v;
+    int64_t pool_layer_stride;   // elements between consecutive layer pools
+    const uint16_t* k;           // [n_layers][rows][H_kv][D]
+    const uint16_t* v;
+    int64_t src_layer_stride;    // rows * H_kv * D
+    const int32_t* page_table;   // [max_seqs][max_pages]
+    int64_t num_pages;
+    int32_t max_pages;
+    int32_t H_kv, D;
+    int32_t n_blocks, n_tiles;
+    int32_t* err;
+    int32_t tile_start[kVarlenMax + 1];  // first tile of block i; tile_start[n_blocks] = n_tiles
+    int32_t seq[kVarlenMax];
+    int32_t first_pos[kVarlenMax];
+    int32_t n_tok[kVarlenMax];
+    int32_t src_row[kVarlenMax];         // packed row of block i's first token
+};
+
 struct AppendArgs {
     uint16_t* pool_k;
     uint16_t* pool_v;
@@ -166,6 +191,7 @@ void set_last_error(const char* msg);
 cudaError_t launch_scatter_i32(int32_t* base, const ScatterI32& s, cudaStream_t st);
 cudaError_t launch_step(const StepPatch& patch, const PlanArgs& plan, cudaStream_t st);
 cudaError_t launch_token_copy(const TokenCopyArgs& a, cudaStream_t st);
+cudaError_t launch_varlen_write(const VarlenWriteArgs& a, int n_layers, cudaStream_t st);
 // Copy each plan entry's page ids from the page table into item_pages
 // ([entries][stride]), so the decode kernel reads them alongside the entry.
 // entries_dev (if non-null) holds the entry count; `entries` is then its bound.

@@ -71,6 +71,7 @@ _SIGS = {
     "kv_seq_info": [_P, _I32, ctypes.POINTER(_I32), _P, _I32, ctypes.POINTER(_I32)],
     "kv_write_tokens": [_P, _I32, _I32, _I32, _I32, _P, _P, _P],
     "kv_read_tokens": [_P, _I32, _I32, _I32, _I32, _P, _P, _P],
+    "kv_write_varlen": [_P, _I32, _I32, _I32, _P, _P, _P, _P, _P, _P],
     "kv_begin_step": [_P, _I32, _P, _P],
     "kv_append": [_P, _I32, _I32, _P, _P, _P],
     "decode_attention": [_P, _I32, _I32, _P, _P, ctypes.c_float, _P],
@@ -197,6 +198,22 @@ def kv_write_tokens(h, layer: int, seq: int, first_pos: int, n: int, k, v, strea
 def kv_read_tokens(h, layer: int, seq: int, first_pos: int, n: int, k_out, v_out, stream=None):
     _check(load().kv_read_tokens(h, layer, seq, first_pos, n, _ptr(k_out), _ptr(v_out), _stream(stream)),
            "kv_read_tokens")
+
+
+def kv_write_varlen(h, layer_first: int, n_layers: int, seq_ids, cu_seqlens, k, v, first_pos=None, stream=None):
+    """Packed varlen bulk write: block i = rows cu_seqlens[i]..cu_seqlens[i+1]-1
+    of k, v ([n_layers][rows][H_kv][d] bf16, device) -> positions
+    first_pos[i].. of sequence seq_ids[i] (first_pos None: all 0)."""
+    ids = _i32_array(seq_ids)
+    cu = _i32_array(cu_seqlens)
+    if len(cu) != len(ids) + 1:
+        raise ValueError("cu_seqlens needs len(seq_ids) + 1 entries")
+    fp = _i32_array(first_pos) if first_pos is not None else None
+    if fp is not None and len(fp) != len(ids):
+        raise ValueError("first_pos needs len(seq_ids) entries")
+    _check(load().kv_write_varlen(h, layer_first, n_layers, len(ids), ctypes.addressof(ids),
+                                  ctypes.addressof(fp) if fp is not None else None, ctypes.addressof(cu),
+                                  _ptr(k), _ptr(v), _stream(stream)), "kv_write_varlen")
 
 
 def kv_begin_step(h, seq_ids, stream=None):

@@ -209,6 +209,26 @@ def kv_block(cfg: WorkloadConfig, layer: int, seq_index: int, n_tokens: int, kin
                  _mix(cfg.seed, 11, layer, seq_index, code), device)
 
 
+def packed_prefix(cfg: WorkloadConfig, layers, lens, device="cpu"):
+    """The cached prefixes of a batch packed for one varlen bulk write:
+    (k, v, cu_seqlens) with k, v bf16 [len(layers)][sum(lens)][H_kv][d] whose
+    rows cu_seqlens[b] .. cu_seqlens[b+1]-1 in slab i are kv_block(cfg,
+    layers[i], b, lens[b]); sequences in batch order."""
+    import torch
+    cu = [0]
+    for n in lens:
+        cu.append(cu[-1] + int(n))
+    shape = (len(layers), cu[-1], cfg.num_kv_heads, cfg.head_dim)
+    k = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    v = torch.empty(shape, dtype=torch.bfloat16, device=device)
+    for i, layer in enumerate(layers):
+        for b, n in enumerate(lens):
+            if int(n):
+                k[i, cu[b]:cu[b + 1]] = kv_block(cfg, layer, b, int(n), "k", device)
+                v[i, cu[b]:cu[b + 1]] = kv_block(cfg, layer, b, int(n), "v", device)
+    return k, v, cu
+
+
 def step_inputs(cfg: WorkloadConfig, step: int, layer: int, device="cpu"):
     """(q [B, H_q, d], k_new [B, H_kv, d], v_new [B, H_kv, d]) bf16 for one
     decode step of one logical layer."""

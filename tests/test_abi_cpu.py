@@ -24,7 +24,7 @@ def test_header_declares_the_boundary(kvlib):
     names = declared_functions()
     for required in ("kv_cache_create", "kv_append", "decode_attention", "kv_cache_destroy"):
         assert required in names
-    assert len(names) == 22
+    assert len(names) == 23
 
 
 def test_library_exports_every_declared_symbol(kvlib):
@@ -61,6 +61,38 @@ def test_data_and_attention_calls_refuse_host_only_caches(kvlib):
         kvlib.kv_append(h, 0, 1, 16, 16)
     with pytest.raises(kvlib.KVDecodeError):
         kvlib.decode_attention(h, 0, 1, 16, 16)
+    kvlib.kv_cache_destroy(h)
+
+
+def test_varlen_write_checks_its_blocks(kvlib):
+    """kv_write_varlen validates every block before it touches the device:
+    positions inside the reserved length, cu_seqlens starting at 0 and not
+    decreasing, no two blocks on one position; a valid call on a host-only
+    cache gets as far as the device check."""
+    h = host_cache(kvlib)
+    a, b = kvlib.kv_seq_create(h), kvlib.kv_seq_create(h)
+    kvlib.kv_seq_reserve(h, a, 40)
+    kvlib.kv_seq_reserve(h, b, 20)
+
+    def code(ids, cu, fp=None, k=16, v=16):
+        with pytest.raises(kvlib.KVDecodeError) as ei:
+            kvlib.kv_write_varlen(h, 0, 1, ids, cu, k, v, first_pos=fp)
+        return ei.value.code, kvlib.load().kv_last_error().decode()
+
+    host_only = (kvlib.KVC_ERR_INVALID, "kv_write_varlen: cache was created host-only")
+    assert code([a, b], [0, 40, 60]) == host_only
+    assert code([a, a, b], [0, 10, 40, 60], fp=[0, 10, 0]) == host_only       # adjacent, no overlap
+    assert code([a, a], [0, 10, 10], fp=[30, 5]) == host_only                  # an empty block is skipped
+    assert "reserved length" in code([a, b], [0, 40, 61])[1]
+    assert "reserved length" in code([a], [0, 5], fp=[36])[1]
+    assert "cu_seqlens[0]" in code([a], [1, 5])[1]
+    assert "must not decrease" in code([a, b], [0, 10, 5])[1]
+    assert "overlap" in code([a, a], [0, 10, 20], fp=[0, 9])[1]
+    assert "overlap" in code([a, a, a], [0, 10, 10, 12], fp=[0, 5, 6])[1]     # empty block between
+    assert "aligned" in code([a], [0, 4], k=8)[1]
+    with pytest.raises(kvlib.KVDecodeError):
+        kvlib.kv_write_varlen(h, 1, 2, [a], [0, 4], 16, 16)                    # layers past the cache
+    kvlib.kv_write_varlen(h, 0, 1, [], [0], None, None)                        # nothing to write
     kvlib.kv_cache_destroy(h)
 
 
