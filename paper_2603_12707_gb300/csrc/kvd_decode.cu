@@ -355,6 +355,72 @@ __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanE
     __syncwarp();
 }
 
+// Merge pass.  SPLIT warps merge a split row's items for one query head
+// h = g * G + hh of batch row b, each owning D / SPLIT dims:
+//     M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c,
+// lane c holding item c's (m, l) and every lane D / (32 * SPLIT) dims of o.
+// All loads (m, l and the o of every item, at most kMaxChunks) are issued
+// before the first use, so a unit costs one round trip to L2.
+constexpr int kMergeSplit = 1;   // warps per (row, query head)
+constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
+
+template <int D>
+__device__ __forceinline__ void merge_unit(const DecodeParams& p, int b, int g, int hh, int part, int lane)
+{
+    constexpr int PER = D / (32 * kMergeSplit);
+    static_assert(PER == 1 || PER == 2 || PER == 4, "dims per lane");
+    const int2 row = p.rows[b];
+    const int nch = row.y;
+    auto slot = [&](int c) { return ((int64_t)(row.x + c) * p.H_kv + g) * p.G + hh; };
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (lane < nch) ml = __ldcg(&p.part_ml[slot(lane)]);
+    const int d0 = part * (D / kMergeSplit) + lane * PER;
+    float vals[kMaxChunks][PER];
+#pragma unroll
+    for (int c = 0; c < kMaxChunks; ++c) {
+        const float* src = p.part_o + slot(c < nch ? c : 0) * D + d0;
+        if (c < nch) {
+            if constexpr (PER == 4) {
+                const float4 t = __ldcg(reinterpret_cast<const float4*>(src));
+                vals[c][0] = t.x; vals[c][1] = t.y; vals[c][2] = t.z; vals[c][3] = t.w;
+            } else if constexpr (PER == 2) {
+                const float2 t = __ldcg(reinterpret_cast<const float2*>(src));
+                vals[c][0] = t.x; vals[c][1] = t.y;
+            } else {
+                vals[c][0] = __ldcg(src);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < PER; ++j) vals[c][j] = 0.f;
+        }
+    }
+    float M = ml.x;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float e = (lane < nch) ? ex2(ml.x - M) : 0.f;
+    float L = e * ml.y;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    const float wgt = e / L;
+    float acc[PER];
+#pragma unroll
+    for (int j = 0; j < PER; ++j) acc[j] = 0.f;
+#pragma unroll
+    for (int c = 0; c < kMaxChunks; ++c) {
+        const float wc = __shfl_sync(0xffffffffu, wgt, c);
+#pragma unroll
+        for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[c][j], acc[j]);
+    }
+    uint16_t* orow = p.out + ((int64_t)b * p.H_q + g * p.G + hh) * D + d0;
+    if constexpr (PER == 4) {
+        *reinterpret_cast<uint2*>(orow) = make_uint2(pack_bf16(acc[0], acc[1]), pack_bf16(acc[2], acc[3]));
+    } else if constexpr (PER == 2) {
+        *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0], acc[1]);
+    } else {
+        orow[0] = (uint16_t)(pack_bf16(acc[0], 0.f) & 0xffffu);
+    }
+}
+
 template <int D, bool GQA, bool FUSED>
 __global__ void __launch_bounds__(kWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
@@ -504,14 +570,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     }
 }
 
-// Second pass.  A split row's (row b, query head h) is merged by SPLIT warps,
-// each owning D/SPLIT dims: lane c < n_chunks holds item c's (m, l); the
-// weights 2^(m_c - M) / sum_c 2^(m_c - M) l_c stay in registers and are
-// broadcast while the lanes (D/SPLIT/32 dims each) accumulate the items' o,
-// sixteen items in flight at a time.
-constexpr int kMergeWarps = 4;
-constexpr int kMergeSplit = 2;
-
+// Second pass: kMergeSplit warps per (row, query head) of a split row.
 template <int D>
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodeParams p, int pdl)
 {
@@ -519,65 +578,15 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
         griddep_launch_dependents();   // the next layer may start streaming now
         griddep_wait();                // the split pass of this layer is complete
     }
-    constexpr int DW = D / kMergeSplit;   // dims per warp
-    constexpr int PER = DW / 32;          // dims per lane
-    constexpr int U = 16;
     const int lane = threadIdx.x & 31;
     const int total = p.batch * p.H_q * kMergeSplit;
     for (int w = blockIdx.x * kMergeWarps + (threadIdx.x >> 5); w < total; w += gridDim.x * kMergeWarps) {
         const int part = w % kMergeSplit;
         const int bh = w / kMergeSplit;
         const int b = bh / p.H_q, h = bh - b * p.H_q;
-        const int2 row = p.rows[b];
-        const int nch = row.y;
-        if (nch <= 1) continue;
-        const int g = h / p.G, hh = h - g * p.G;
-        auto slot = [&](int c) { return ((int64_t)(row.x + c) * p.H_kv + g) * p.G + hh; };
-        float m = -INFINITY, l = 0.f;
-        if (lane < nch) {
-            const float2 ml = __ldcg(&p.part_ml[slot(lane)]);
-            m = ml.x;
-            l = ml.y;
-        }
-        float M = m;
-#pragma unroll
-        for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-        const float e = (lane < nch) ? ex2(m - M) : 0.f;
-        float L = e * l;
-#pragma unroll
-        for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-        const float wgt = e / L;
-        const int d0 = part * DW + lane * PER;
-        float acc[PER];
-#pragma unroll
-        for (int k = 0; k < PER; ++k) acc[k] = 0.f;
-        for (int c0 = 0; c0 < nch; c0 += U) {
-            float v[U][PER];
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const int c = c0 + u;
-                const float* po = p.part_o + slot(c < nch ? c : 0) * D + d0;
-                if constexpr (PER == 2) {
-                    const float2 t = __ldcg(reinterpret_cast<const float2*>(po));
-                    v[u][0] = t.x; v[u][1] = t.y;
-                } else {
-                    v[u][0] = __ldcg(po);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
-                if (c0 + u < nch)
-#pragma unroll
-                    for (int k = 0; k < PER; ++k) acc[k] = fmaf(wc, v[u][k], acc[k]);
-            }
-        }
-        uint16_t* orow = p.out + ((int64_t)b * p.H_q + h) * D + d0;
-        if constexpr (PER == 2) {
-            *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0], acc[1]);
-        } else {
-            orow[0] = (uint16_t)(pack_bf16(acc[0], 0.f) & 0xffffu);
-        }
+        if (p.rows[b].y <= 1) continue;
+        const int g = h / p.G;
+        merge_unit<D>(p, b, g, h - g * p.G, part, lane);
     }
 }
 
@@ -632,7 +641,7 @@ cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cu
 {
     const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
-                                                                   (int64_t)num_sms * 16));
+                                                                   (int64_t)num_sms * 32));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(kMergeWarps * 32);
