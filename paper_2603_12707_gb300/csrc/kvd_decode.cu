@@ -363,6 +363,8 @@ __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanE
 // before the first use, so a unit costs one round trip to L2.
 constexpr int kMergeSplit = 1;   // warps per (row, query head)
 constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
+constexpr int kMergeBatch = 32;  // items whose o is loaded before the first use
+constexpr int kMergeGridPerSm = 32;   // merge CTAs per SM at most (one-warp CTAs)
 
 template <int D>
 __device__ __forceinline__ void merge_unit(const DecodeParams& p, int b, int g, int hh, int part, int lane)
@@ -375,25 +377,29 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int b, int g, 
     float2 ml = make_float2(-INFINITY, 0.f);
     if (lane < nch) ml = __ldcg(&p.part_ml[slot(lane)]);
     const int d0 = part * (D / kMergeSplit) + lane * PER;
-    float vals[kMaxChunks][PER];
+    float vals[kMergeBatch][PER];
+    auto load = [&](int c0) {
 #pragma unroll
-    for (int c = 0; c < kMaxChunks; ++c) {
+    for (int u = 0; u < kMergeBatch; ++u) {
+        const int c = c0 + u;
         const float* src = p.part_o + slot(c < nch ? c : 0) * D + d0;
         if (c < nch) {
             if constexpr (PER == 4) {
                 const float4 t = __ldcg(reinterpret_cast<const float4*>(src));
-                vals[c][0] = t.x; vals[c][1] = t.y; vals[c][2] = t.z; vals[c][3] = t.w;
+                vals[u][0] = t.x; vals[u][1] = t.y; vals[u][2] = t.z; vals[u][3] = t.w;
             } else if constexpr (PER == 2) {
                 const float2 t = __ldcg(reinterpret_cast<const float2*>(src));
-                vals[c][0] = t.x; vals[c][1] = t.y;
+                vals[u][0] = t.x; vals[u][1] = t.y;
             } else {
-                vals[c][0] = __ldcg(src);
+                vals[u][0] = __ldcg(src);
             }
         } else {
 #pragma unroll
-            for (int j = 0; j < PER; ++j) vals[c][j] = 0.f;
+            for (int j = 0; j < PER; ++j) vals[u][j] = 0.f;
         }
     }
+    };
+    load(0);
     float M = ml.x;
 #pragma unroll
     for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
@@ -405,11 +411,14 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int b, int g, 
     float acc[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) acc[j] = 0.f;
+    for (int c0 = 0; c0 < nch; c0 += kMergeBatch) {
+        if (c0) load(c0);
 #pragma unroll
-    for (int c = 0; c < kMaxChunks; ++c) {
-        const float wc = __shfl_sync(0xffffffffu, wgt, c);
+        for (int u = 0; u < kMergeBatch; ++u) {
+            const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
 #pragma unroll
-        for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[c][j], acc[j]);
+            for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[u][j], acc[j]);
+        }
     }
     uint16_t* orow = p.out + ((int64_t)b * p.H_q + g * p.G + hh) * D + d0;
     if constexpr (PER == 4) {
@@ -637,11 +646,23 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
 
 }  // namespace
 
+// The merge pass uses no shared memory; asking for the largest shared-memory
+// carveout keeps an SM that hosts its CTAs in the configuration of the split
+// pass, so the next layer's split-pass CTAs can still be placed there.
+template <int D>
+cudaError_t prepare_merge()
+{
+    static cudaError_t status =
+        cudaFuncSetAttribute(merge_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    return status;
+}
+
 cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st)
 {
+    if (cudaError_t e = D == 128 ? prepare_merge<128>() : prepare_merge<64>()) return e;
     const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
-                                                                   (int64_t)num_sms * 32));
+                                                                   (int64_t)num_sms * kMergeGridPerSm));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(kMergeWarps * 32);
