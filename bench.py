@@ -134,9 +134,11 @@ def gpu_smi_id(torch, dev):
 
 
 # --------------------------------------------------------- kernel traffic
-def committed_traffic(kernel_src):
-    """DRAM bytes per launch of the decode kernel from the committed ncu
-    summary, valid only if it was taken on the current kernel source."""
+def committed_traffic(kernel_src, workload, algorithmic_bytes):
+    """DRAM bytes per launch of the decode kernel: the committed ncu capture's
+    traffic / algorithmic ratio for this workload times this launch's
+    algorithmic bytes; None unless the capture was taken on the current
+    kernel source."""
     p = os.path.join(ROOT, "profiles", "decode_kernel_traffic.json")
     if not os.path.exists(p):
         return None
@@ -144,7 +146,10 @@ def committed_traffic(kernel_src):
         d = json.load(f)
     with open(kernel_src, "rb") as f:
         h = hashlib.sha256(f.read()).hexdigest()[:16]
-    return d if d.get("source_sha256_16") == h else None
+    cap = d.get("captures", {}).get(workload)
+    if d.get("source_sha256_16") != h or cap is None:
+        return None
+    return int(round(cap["traffic_over_algorithmic"] * algorithmic_bytes))
 
 
 # ------------------------------------------------------------- CPU oracle
@@ -529,7 +534,8 @@ def main():
     attn_bytes = statistics.mean(r["attn_bytes"])
     peak, peak_kind = measured_peaks()
     achieved = attn_bytes / (attn_ms / 1e3) / 1e9
-    traffic = committed_traffic(os.path.join(ROOT, "paper_2603_12707_gb300", "csrc", "kvd_decode.cu"))
+    traffic = None if args.unfused else committed_traffic(
+        os.path.join(ROOT, "paper_2603_12707_gb300", "csrc", "kvd_decode.cu"), cfg.name, attn_bytes)
     out = {
         "metric": METRIC, "value": round(gbs, 2), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
@@ -544,7 +550,7 @@ def main():
         "roofline": {"bound": "hbm", "kernel": "decode_attention" if args.unfused else "decode_attention_append",
                      "achieved": round(achieved, 2),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "traffic": (traffic["dram_bytes_per_launch_full"] if traffic else None),
+                     "traffic": traffic,
                      "algorithmic_bytes_per_launch": int(attn_bytes), "avg_launch_ms": round(attn_ms, 4)},
         "clocks": r["clocks"],
         "gpu_launches": r["launches"],
