@@ -448,11 +448,18 @@ def varlen_main(args, rank, world):
 
 
 def reduce_max(torch, x, world):
+    """Max of x over the ranks (the job's time is its slowest rank's)."""
     if world == 1:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cpu" if torch.distributed.get_backend() == "gloo" else "cuda"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_gbs(bytes_per_rank, max_ms, world):
+    """Whole-job throughput: every rank's bytes over the slowest rank's time."""
+    return bytes_per_rank * world / (max_ms / 1e3) / 1e9
 
 
 def main():
@@ -527,8 +534,7 @@ def main():
     r = run_gpu(args, rank, world)
     cfg, L = r["cfg"], r["L"]
     ms = reduce_max(torch, r["ms"], world)
-    total_bytes = sum(r["step_bytes"]) * world
-    gbs = total_bytes / (ms / 1e3) / 1e9
+    gbs = whole_job_gbs(sum(r["step_bytes"]), ms, world)
     steps_per_s = args.steps / (ms / 1e3)
     attn_ms = statistics.mean(r["attn_ms"])
     attn_bytes = statistics.mean(r["attn_bytes"])
