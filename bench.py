@@ -1,8 +1,12 @@
 """Decode-step benchmark: paged decode attention (+ fused K/V append) on GB300.
 
-A step is one pass of the whole hot path over one batch: kv_begin_step (lazy
-page allocation, page-table update and split plan on the device) and, for each
-of the L layers, kv_append then decode_attention.  The default workload is the
+A step is one pass of the whole hot path over one batch: the step's lazy page
+allocation, page-table update and split plan (kv_begin_step_device, all on the
+device) and, for each of the L layers, the fused K/V append + decode attention
+(decode_attention_append; the merge pass follows when a row is split).  By
+default the step is captured once into CUDA graphs and replayed; --host-steps
+plans on the host (kv_begin_step) and launches from Python, --unfused launches
+kv_append and decode_attention separately.  The default workload is the
 LLaVA-1.5-7B-shaped batch (32 layers, 32/32 heads, d 128, batch 64, 576 vision
 tokens + U[64,512] prompt + U{0..256} generated tokens, page 16, shuffled page
 table).  Inputs are seeded synthetic draws (paper_2603_12707_gb300.workloads).
@@ -475,15 +479,15 @@ def main():
                     help="target pages per work item (0: the library's automatic choice)")
     ap.add_argument("--unfused", action="store_true",
                     help="kv_append and decode_attention as two launches per layer (default: one fused launch)")
-    ap.add_argument("--graph", action="store_true",
-                    help="replay each step from CUDA graphs (device-side kv_begin_step, fused layers)")
+    ap.add_argument("--host-steps", action="store_true",
+                    help="plan each step on the host (kv_begin_step) and launch the layers from Python "
+                         "(default: replay CUDA graphs of kv_begin_step_device and the fused layers)")
     ap.add_argument("--varlen-write", action="store_true",
                     help="time the packed varlen bulk K/V write of the workload's prefixes instead of decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     args = ap.parse_args()
-    if args.graph and args.unfused:
-        ap.error("--graph captures the fused layers; drop --unfused")
+    args.graph = not (args.host_steps or args.unfused)
     if args.warmup < 3:
         log("warning: fewer than 3 warm-up steps")
 
