@@ -138,6 +138,16 @@ def gpu_smi_id(torch, dev):
 
 
 # --------------------------------------------------------- kernel traffic
+def kernel_code_hash(path):
+    """sha256 (16 hex digits) of a source file's code: line comments, blank
+    lines and surrounding whitespace removed, so a comment edit keeps a
+    capture valid and any code edit voids it."""
+    import re
+    with open(path) as f:
+        lines = [re.sub(r"//.*$", "", l).strip() for l in f]
+    return hashlib.sha256("\n".join(l for l in lines if l).encode()).hexdigest()[:16]
+
+
 def committed_traffic(kernel_src, workload, algorithmic_bytes):
     """DRAM bytes per launch of the decode kernel: the committed ncu capture's
     traffic / algorithmic ratio for this workload times this launch's
@@ -148,8 +158,7 @@ def committed_traffic(kernel_src, workload, algorithmic_bytes):
         return None
     with open(p) as f:
         d = json.load(f)
-    with open(kernel_src, "rb") as f:
-        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    h = kernel_code_hash(kernel_src)
     cap = d.get("captures", {}).get(workload)
     if d.get("source_sha256_16") != h or cap is None:
         return None

@@ -3,15 +3,17 @@
 // Schedule.  A step's plan cuts every (sequence, KV head) into work items of
 // consecutive pages.  A persistent grid of warps pulls items from a global
 // counter; each warp runs its items independently:
-//   * one lane streams (page, head) tiles of K and V into the warp's private
-//     ring of R shared-memory stages with 2-D TMA tile loads (128-byte
-//     swizzle, L2 evict-first), completing on one mbarrier per stage;
+//   * one lane streams the (page, head) tiles of K and V into the warp's
+//     private ring of R shared-memory stages, one 4-D TMA tile load per page
+//     covering K and V (128-byte swizzle, L2 evict-first), completing on one
+//     mbarrier per stage;
 //   * the warp computes an online softmax over the item's tokens for the G
 //     query heads of the KV head (running max m in log2 units, running sum l,
 //     unnormalised accumulator o, all fp32);
 //   * a row with one item writes bf16 output directly; otherwise each item
 //     stores (o, m, l) as a partial and a second pass (merge_kernel, one warp
-//     per (row, query head), one lane per item) merges them by log-sum-exp:
+//     per (row, query head), one lane per item's (m, l), every item's o in
+//     flight at once) merges them by log-sum-exp:
 //         M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c.
 // MHA (G = 1, 1 flop per byte) runs on the CUDA cores; GQA (2 <= G <= 8) runs
 // Q.K^T and P.V as m16n8k16 bf16 MMAs with the 16 tokens of a page as M and the
