@@ -325,20 +325,29 @@ def run_gpu(args, rank, world):
     if graphs is not None:
         kd.kv_cache_device_steps(sess.h, B, False, stream)   # host-driven steps from here on
 
-    # ---- end to end: host inputs -> device -> host outputs, every step
+    # ---- end to end: host inputs -> device -> host outputs, every step.
+    # A step's q, k_new, v_new of all layers sit in one pinned host buffer
+    # and go over in one copy; all layers' outputs come back in one copy.
     e2e = None
     if not args.no_e2e:
-        pin = lambda t: t.cpu().pin_memory()
-        hq = [pin(q) for q in qs]
-        hk = [pin(k) for k in ks]
-        hv = [pin(v) for v in vs]
-        ho = [torch.empty_like(o, device="cpu").pin_memory() for o in outs]
-        dq = [torch.empty_like(q) for q in qs]
-        dk = [torch.empty_like(k) for k in ks]
-        dv = [torch.empty_like(v) for v in vs]
+        Hq, Hkv, d = cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+        per_layer = B * (Hq + 2 * Hkv) * d
+        h_in = torch.empty(L * per_layer, dtype=torch.bfloat16).pin_memory()
+        for l in range(L):
+            h_in[l * per_layer:(l + 1) * per_layer] = torch.cat(
+                [qs[l].reshape(-1), ks[l].reshape(-1), vs[l].reshape(-1)]).cpu()
+        d_in = torch.empty_like(h_in, device="cuda")
+        d_out = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device="cuda")
+        h_out = torch.empty_like(d_out, device="cpu").pin_memory()
+
+        def views(l):
+            x = d_in[l * per_layer:(l + 1) * per_layer]
+            return (x[:B * Hq * d].view(B, Hq, d), x[B * Hq * d:B * (Hq + Hkv) * d].view(B, Hkv, d),
+                    x[B * (Hq + Hkv) * d:].view(B, Hkv, d))
+
         e_bytes = 0
-        h2d = sum(t.numel() * 2 for t in hq + hk + hv)
-        d2h = sum(t.numel() * 2 for t in ho)
+        h2d = h_in.numel() * 2
+        d2h = h_out.numel() * 2
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         torch.cuda.synchronize()
         if world > 1:
@@ -350,18 +359,16 @@ def run_gpu(args, rank, world):
                 att = [int(n) + 1 for n in sess.lens]
                 a, p = layer_bytes(cfg, att)
                 e_bytes += L * (a + p)
-                for l in range(L):
-                    dq[l].copy_(hq[l], non_blocking=True)
-                    dk[l].copy_(hk[l], non_blocking=True)
-                    dv[l].copy_(hv[l], non_blocking=True)
+                d_in.copy_(h_in, non_blocking=True)
                 sess.begin_step()
                 for l in range(L):
+                    q, k, v = views(l)
                     if args.unfused:
-                        sess.append(l, dk[l], dv[l])
-                        sess.attend(l, dq[l], outs[l])
+                        sess.append(l, k, v)
+                        sess.attend(l, q, d_out[l])
                     else:
-                        sess.append_attend(l, dq[l], dk[l], dv[l], outs[l])
-                    ho[l].copy_(outs[l], non_blocking=True)
+                        sess.append_attend(l, q, k, v, d_out[l])
+                h_out.copy_(d_out, non_blocking=True)
             s1.record(stream)
         stream.synchronize()
         wall = time.perf_counter() - w0
