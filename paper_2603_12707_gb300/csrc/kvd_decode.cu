@@ -622,7 +622,7 @@ cudaError_t variant_info(DecodeVariant* v)
 }
 
 template <int D, bool GQA>
-cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+cudaError_t launch_variant(bool fused, bool pdl, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
                            const DecodeParams& p, cudaStream_t st)
 {
     if (!fused) {
@@ -642,7 +642,7 @@ cudaError_t launch_variant(bool fused, int grid, const CUtensorMap& tk, const CU
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, decode_kernel<D, GQA, true>, tk, tv, p);
 }
 
@@ -688,13 +688,13 @@ cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v)
     return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_decode(int D, bool gqa, bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
-                          const DecodeParams& p, cudaStream_t st)
+cudaError_t launch_decode(int D, bool gqa, bool fused, bool pdl, int grid, const CUtensorMap& tk,
+                          const CUtensorMap& tv, const DecodeParams& p, cudaStream_t st)
 {
-    if (D == 128) return gqa ? launch_variant<128, true>(fused, grid, tk, tv, p, st)
-                             : launch_variant<128, false>(fused, grid, tk, tv, p, st);
-    if (D == 64) return gqa ? launch_variant<64, true>(fused, grid, tk, tv, p, st)
-                            : launch_variant<64, false>(fused, grid, tk, tv, p, st);
+    if (D == 128) return gqa ? launch_variant<128, true>(fused, pdl, grid, tk, tv, p, st)
+                             : launch_variant<128, false>(fused, pdl, grid, tk, tv, p, st);
+    if (D == 64) return gqa ? launch_variant<64, true>(fused, pdl, grid, tk, tv, p, st)
+                            : launch_variant<64, false>(fused, pdl, grid, tk, tv, p, st);
     return cudaErrorInvalidValue;
 }
 

@@ -95,6 +95,11 @@ struct kv_cache {
     uint32_t* queue = nullptr;                  // two (next item, warps done) counter pairs
     uint32_t fused_launches = 0;                // fused launches alternate counter pairs
     int64_t launches = 0;                       // kernels launched (reported by kv_cache_query)
+    // A fused launch may depend programmatically on the launch before it only
+    // if that was an attention launch on the same stream: its early reads
+    // (plan, page lists, cached pages) must not race any other writer.
+    int64_t chain_launches = -1;                // `launches` right after the last attention launch
+    void* chain_stream = nullptr;
     int32_t* err = nullptr;
     PlanEntry* plan = nullptr;
     int64_t plan_cap = 0;
@@ -818,7 +823,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     const int64_t want = (p.n_items + c->variant.warps - 1) / c->variant.warps;
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
     p.kv_map = 1;
-    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, grid, c->tmaps[layer], c->tmaps[layer], p,
+    const bool pdl = fused && c->chain_launches == c->launches && c->chain_stream == stream;
+    KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, pdl, grid, c->tmaps[layer], c->tmaps[layer], p,
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
     if (c->step_split) {
@@ -826,6 +832,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
         ++c->launches;
     }
     if (fused) ++c->fused_launches;
+    c->chain_launches = c->launches;
+    c->chain_stream = stream;
     return KVC_OK;
 }
 

@@ -216,7 +216,7 @@ cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cu
 // fused: the append + attention kernel, launched with programmatic dependent
 // launch (it streams its first pages before the previous kernel finishes and
 // reads q / k_new / v_new and writes anything only after it has).
-cudaError_t launch_decode(int D, bool gqa, bool fused, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
+cudaError_t launch_decode(int D, bool gqa, bool fused, bool pdl, int grid, const CUtensorMap& tk, const CUtensorMap& tv,
                           const DecodeParams& p, cudaStream_t st);
 
 }  // namespace kvd

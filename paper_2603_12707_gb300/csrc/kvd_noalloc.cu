@@ -270,7 +270,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     const int64_t resident = (int64_t)num_sms * std::max(1, var.ctas_per_sm);
     const int64_t want = (p.n_items + var.warps - 1) / var.warps;
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
-    if (cudaError_t e = launch_decode(head_dim, G > 1, false, grid, maps[0], maps[1], p, st); e != cudaSuccess)
+    if (cudaError_t e = launch_decode(head_dim, G > 1, false, false, grid, maps[0], maps[1], p, st); e != cudaSuccess)
         return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     if (split_rows)
         if (cudaError_t e = launch_merge(head_dim, false, num_sms, p, st); e != cudaSuccess)
