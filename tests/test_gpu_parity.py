@@ -265,3 +265,66 @@ def test_decode_matches_oracle_full_size(name, layers, rows):
         ref, vmax = t.oracle(layer, q, rows=r)
         assert_close(bf16_to_f64(out)[r], ref, vmax, gqa=cfg.group > 1, what=(name, layer))
     t.close()
+
+
+# -------------------------------- full size, in the bench's launch configuration
+FULL_GRAPH = [
+    # config, logical layers checked (distinct pools; for the ragged config the
+    # last logical layer of each checked pool), sampled batch rows
+    ("llava", [0, 31], [0, 1, 63]),
+    ("qwen", [0, 27], [0, 5, 31]),
+    ("long", [0, 27], [0, 7]),
+    ("ragged", [24, 31], [0, 100, 255]),
+]
+
+
+@pytest.mark.parametrize("name,layers,rows", FULL_GRAPH)
+def test_graph_replayed_steps_match_oracle_full_size(name, layers, rows):
+    """Device-side steps and all L fused layers captured into CUDA graphs and
+    replayed, as bench.py times them; after one eager and three replayed
+    steps every checked layer's output matches the oracle over the prefix
+    plus the four appended tokens."""
+    cfg = wl.CONFIGS[name]
+    L, B = cfg.num_layers, cfg.batch
+    phys = sorted({l % cfg.phys_layers for l in layers})
+    assert len(phys) == len(layers)
+    t = Tracked(cfg, extra_tokens=8, layers_filled=phys, keep_rows=rows)
+    sess = t.sess
+    s = torch.cuda.Stream()
+    ins = [wl.step_inputs(cfg, 0, l, "cuda") for l in range(L)]
+    outs = [torch.empty_like(i[0]) for i in ins]
+    ids = torch.tensor(sess.seq_ids, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    kd.kv_cache_device_steps(sess.h, B, True, s)
+
+    def all_layers():
+        for l in range(L):
+            kd.decode_attention_append(sess.h, sess.phys(l), B, ins[l][0], ins[l][1], ins[l][2], outs[l], 0.0, s)
+
+    with torch.cuda.stream(s):
+        kd.kv_begin_step_device(sess.h, B, ids, s)
+        all_layers()
+    s.synchronize()
+    g_step, g_layers = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_step, stream=s):
+        kd.kv_begin_step_device(sess.h, B, ids, s)
+    with torch.cuda.graph(g_layers, stream=s):
+        all_layers()
+    with torch.cuda.stream(s):
+        for _ in range(3):
+            g_step.replay()
+            g_layers.replay()
+    s.synchronize()
+    steps = 4
+    kd.kv_cache_sync(sess.h)
+    for b in rows:
+        assert kd.kv_seq_info(sess.h, sess.seq_ids[b])[0] == int(sess.lens0[b]) + steps
+    for l in layers:
+        p = sess.phys(l)
+        kh, vh = u16(ins[l][1]), u16(ins[l][2])
+        for b in rows:
+            t.k[(p, b)] += [kh[b]] * steps
+            t.v[(p, b)] += [vh[b]] * steps
+        ref, vmax = t.oracle(l, ins[l][0], rows=rows)
+        assert_close(bf16_to_f64(outs[l])[rows], ref, vmax, gqa=cfg.group > 1, what=(name, l))
+    t.close()
