@@ -14,7 +14,7 @@ from paper_2603_12707_gb300 import kvdecode as kd
 from paper_2603_12707_gb300 import workloads as wl
 from paper_2603_12707_gb300.harness import DecodeSession
 
-from _gpu_common import _CAI, u16
+from _gpu_common import _CAI, assert_close, bf16_to_f64, u16
 
 pytestmark = pytest.mark.gpu
 
@@ -127,4 +127,35 @@ def test_varlen_write_llava_handoff(kvlib):
             pt = np.asarray(kd.kv_seq_info(sess.h, s)[1], dtype=np.int32)
             assert np.array_equal(oracle.kv_gather(pk, pt, 0, lens[b]), src_k[cu[b]:cu[b + 1]]), (l, b)
             assert np.array_equal(oracle.kv_gather(pv, pt, 0, lens[b]), src_v[cu[b]:cu[b + 1]]), (l, b)
+    sess.close()
+
+
+def test_decode_after_varlen_prefix_matches_oracle(kvlib):
+    """The prefixes of a ragged GQA batch written by one kv_write_varlen call
+    (all layers), then three fused decode steps: every output matches the
+    oracle over the written prefix plus the appended tokens."""
+    cfg = wl.custom("varlen_decode", 3, 28, 4, 128, 5, lens=[1, 16, 17, 300, 1000], seed=77,
+                    page_order="shuffled")
+    sess = DecodeSession(cfg, extra_tokens=4)
+    lens = [int(n) for n in sess.lens0]
+    k, v, cu = wl.packed_prefix(cfg, range(cfg.num_layers), lens, "cuda")
+    kd.kv_write_varlen(sess.h, 0, cfg.num_layers, sess.seq_ids, cu, k, v)
+    hk = {(l, b): list(u16(k[l, cu[b]:cu[b + 1]])) for l in range(cfg.num_layers) for b in range(cfg.batch)}
+    hv = {(l, b): list(u16(v[l, cu[b]:cu[b + 1]])) for l in range(cfg.num_layers) for b in range(cfg.batch)}
+    for step in range(3):
+        sess.begin_step()
+        for l in range(cfg.num_layers):
+            q, kn, vn = wl.step_inputs(cfg, step, l, "cuda")
+            out = torch.empty_like(q)
+            sess.append_attend(l, q, kn, vn, out)
+            torch.cuda.synchronize()
+            for b in range(cfg.batch):
+                hk[(l, b)].append(u16(kn)[b])
+                hv[(l, b)].append(u16(vn)[b])
+            kk = np.concatenate([np.stack(hk[(l, b)]) for b in range(cfg.batch)])
+            vv = np.concatenate([np.stack(hv[(l, b)]) for b in range(cfg.batch)])
+            ref = oracle.decode_attention(u16(q), [len(hk[(l, b)]) for b in range(cfg.batch)], kk, vv)
+            vmax = np.array([np.abs(oracle.bf16_to_f64(np.stack(hv[(l, b)]))).max() for b in range(cfg.batch)])
+            assert_close(bf16_to_f64(out), ref, vmax, gqa=True, what=(step, l))
+    assert sess.query().device_error == 0
     sess.close()
