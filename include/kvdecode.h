@@ -222,13 +222,15 @@ KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, cons
  * into position s_b of each sequence and used in place of that slot's old
  * contents while the layer's pages stream through shared memory.  Same
  * result and cache contents as kv_append followed by decode_attention.
- * The kernel is launched with programmatic dependent launch: it may start,
- * and stream this layer's cached pages (positions < s_b), while the kernel
- * launched just before it on `stream` is finishing; it reads q, k_new and
- * v_new and writes anything only after that kernel has completed.  So the
- * kernel launched just before it must not write this layer's cached pages
- * (none of this library's kernels does; a foreign kernel could only do so if
- * it signalled its dependents early). */
+ * When the library's previous launch on `stream` was an attention launch
+ * (decode_attention or decode_attention_append of this cache), the kernel is
+ * launched with programmatic dependent launch: it may start, and stream this
+ * layer's cached pages (positions < s_b), while that launch is finishing; it
+ * reads q, k_new and v_new and writes anything only after the kernel before
+ * it has completed.  After any other call of this library it is an ordinary
+ * launch.  So a kernel the caller enqueues between two layers must not write
+ * the cache's pages (a foreign kernel could only race with the early reads
+ * if it signalled its dependents early). */
 KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batch, const void *q,
                                     const void *k_new, const void *v_new, void *out,
                                     float softmax_scale, void *stream);

@@ -1,4 +1,4 @@
-// Inline-PTX helpers for sm_103a: mbarrier, 2-D TMA tile loads, ldmatrix,
+// Inline-PTX helpers for sm_103a: mbarrier, 3-D / 4-D TMA tile loads, ldmatrix,
 // warp-level bf16 MMA, ex2, bf16 packing.
 #pragma once
 
@@ -73,18 +73,6 @@ __device__ __forceinline__ uint64_t l2_policy_evict_first()
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
     return pol;
-}
-
-// 2-D tiled load of box {x, y} (x innermost, in elements) into shared memory,
-// completing `bytes` of transaction count on mbarrier `bar`.
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t x,
-                                            int32_t y, uint32_t bar, uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
-        : "memory");
 }
 
 // 3-D / 4-D tiled loads (coordinates innermost first).
