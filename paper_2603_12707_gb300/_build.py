@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJ = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkvdecode.so")
-SOURCES = ["kvd_host.cpp", "kvd_cache.cu", "kvd_decode.cu", "kvd_noalloc.cu"]
+SOURCES = ["kvd_host.cpp", "kvd_cache.cu", "kvd_decode.cu", "kvd_merge.cu", "kvd_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

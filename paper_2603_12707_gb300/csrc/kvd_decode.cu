@@ -11,7 +11,8 @@
 //     query heads of the KV head (running max m in log2 units, running sum l,
 //     unnormalised accumulator o, all fp32);
 //   * a row with one item writes bf16 output directly; otherwise each item
-//     stores (o, m, l) as a partial and a second pass (merge_kernel, one warp
+//     stores (o, m, l) as a partial and a second pass (merge_kernel in
+//     kvd_merge.cu, one warp
 //     per (row, query head), one lane per item's (m, l), every item's o in
 //     flight at once) merges them by log-sum-exp:
 //         M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c.
@@ -357,81 +358,6 @@ __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanE
     __syncwarp();
 }
 
-// Merge pass.  SPLIT warps merge a split row's items for one query head
-// h = g * G + hh of batch row b, each owning D / SPLIT dims:
-//     M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c,
-// lane c holding item c's (m, l) and every lane D / (32 * SPLIT) dims of o.
-// All loads (m, l and the o of every item, at most kMaxChunks) are issued
-// before the first use, so a unit costs one round trip to L2.
-constexpr int kMergeSplit = 1;   // warps per (row, query head)
-constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
-constexpr int kMergeBatch = 32;  // items whose o is loaded before the first use
-constexpr int kMergeGridPerSm = 32;   // merge CTAs per SM at most (one-warp CTAs)
-
-template <int D>
-__device__ __forceinline__ void merge_unit(const DecodeParams& p, int b, int g, int hh, int part, int lane)
-{
-    constexpr int PER = D / (32 * kMergeSplit);
-    static_assert(PER == 1 || PER == 2 || PER == 4, "dims per lane");
-    const int2 row = p.rows[b];
-    const int nch = row.y;
-    auto slot = [&](int c) { return ((int64_t)(row.x + c) * p.H_kv + g) * p.G + hh; };
-    float2 ml = make_float2(-INFINITY, 0.f);
-    if (lane < nch) ml = __ldcg(&p.part_ml[slot(lane)]);
-    const int d0 = part * (D / kMergeSplit) + lane * PER;
-    float vals[kMergeBatch][PER];
-    auto load = [&](int c0) {
-#pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
-        const int c = c0 + u;
-        const float* src = p.part_o + slot(c < nch ? c : 0) * D + d0;
-        if (c < nch) {
-            if constexpr (PER == 4) {
-                const float4 t = __ldcg(reinterpret_cast<const float4*>(src));
-                vals[u][0] = t.x; vals[u][1] = t.y; vals[u][2] = t.z; vals[u][3] = t.w;
-            } else if constexpr (PER == 2) {
-                const float2 t = __ldcg(reinterpret_cast<const float2*>(src));
-                vals[u][0] = t.x; vals[u][1] = t.y;
-            } else {
-                vals[u][0] = __ldcg(src);
-            }
-        } else {
-#pragma unroll
-            for (int j = 0; j < PER; ++j) vals[u][j] = 0.f;
-        }
-    }
-    };
-    load(0);
-    float M = ml.x;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float e = (lane < nch) ? ex2(ml.x - M) : 0.f;
-    float L = e * ml.y;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    const float wgt = e / L;
-    float acc[PER];
-#pragma unroll
-    for (int j = 0; j < PER; ++j) acc[j] = 0.f;
-    for (int c0 = 0; c0 < nch; c0 += kMergeBatch) {
-        if (c0) load(c0);
-#pragma unroll
-        for (int u = 0; u < kMergeBatch; ++u) {
-            const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
-#pragma unroll
-            for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[u][j], acc[j]);
-        }
-    }
-    uint16_t* orow = p.out + ((int64_t)b * p.H_q + g * p.G + hh) * D + d0;
-    if constexpr (PER == 4) {
-        *reinterpret_cast<uint2*>(orow) = make_uint2(pack_bf16(acc[0], acc[1]), pack_bf16(acc[2], acc[3]));
-    } else if constexpr (PER == 2) {
-        *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[0], acc[1]);
-    } else {
-        orow[0] = (uint16_t)(pack_bf16(acc[0], 0.f) & 0xffffu);
-    }
-}
-
 template <int D, bool GQA, bool FUSED>
 __global__ void __launch_bounds__(kWarps * 32)
     decode_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
@@ -581,26 +507,6 @@ __global__ void __launch_bounds__(kWarps * 32)
     }
 }
 
-// Second pass: kMergeSplit warps per (row, query head) of a split row.
-template <int D>
-__global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodeParams p, int pdl)
-{
-    if (pdl) {
-        griddep_launch_dependents();   // the next layer may start streaming now
-        griddep_wait();                // the split pass of this layer is complete
-    }
-    const int lane = threadIdx.x & 31;
-    const int total = p.batch * p.H_q * kMergeSplit;
-    for (int w = blockIdx.x * kMergeWarps + (threadIdx.x >> 5); w < total; w += gridDim.x * kMergeWarps) {
-        const int part = w % kMergeSplit;
-        const int bh = w / kMergeSplit;
-        const int b = bh / p.H_q, h = bh - b * p.H_q;
-        if (p.rows[b].y <= 1) continue;
-        const int g = h / p.G;
-        merge_unit<D>(p, b, g, h - g * p.G, part, lane);
-    }
-}
-
 template <int D, bool GQA, bool FUSED>
 cudaError_t prepare_variant()
 {
@@ -647,39 +553,6 @@ cudaError_t launch_variant(bool fused, bool pdl, int grid, const CUtensorMap& tk
 }
 
 }  // namespace
-
-// The merge pass uses no shared memory; asking for the largest shared-memory
-// carveout keeps an SM that hosts its CTAs in the configuration of the split
-// pass, so the next layer's split-pass CTAs can still be placed there.
-template <int D>
-cudaError_t prepare_merge()
-{
-    static cudaError_t status =
-        cudaFuncSetAttribute(merge_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    return status;
-}
-
-cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st)
-{
-    if (cudaError_t e = D == 128 ? prepare_merge<128>() : prepare_merge<64>()) return e;
-    const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
-                                                                   (int64_t)num_sms * kMergeGridPerSm));
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(kMergeWarps * 32);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
-    const int flag = pdl ? 1 : 0;
-    if (D == 128) return cudaLaunchKernelEx(&cfg, merge_kernel<128>, p, flag);
-    if (D == 64) return cudaLaunchKernelEx(&cfg, merge_kernel<64>, p, flag);
-    return cudaErrorInvalidValue;
-}
 
 cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v)
 {
