@@ -125,6 +125,7 @@ struct kv_cache {
     bool step_active = false;
     bool step_dev = false;                      // the step's plan was built on the device
     bool step_split = false;                    // some row of the step has several items
+    int32_t step_max_chunks = kMaxChunks;       // bound on the items of a row of the step
     int32_t step_batch = 0;
     int32_t step_entries = 0;
     int32_t split_override = 0;
@@ -676,10 +677,12 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     int64_t entries = 0;
     int32_t stride = 1;
     bool split = false;
+    int32_t max_chunks = 1;
     for (int32_t b = 0; b < batch; ++b) {
         const int nch = row_chunks(np_after[b], T);
         entries += nch;
         split = split || nch > 1;
+        max_chunks = std::max(max_chunks, nch);
         stride = std::max(stride, (np_after[b] + nch - 1) / nch);
     }
     if (!c->host_only)
@@ -740,6 +743,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     c->step_active = true;
     c->step_dev = false;
     c->step_split = split;
+    c->step_max_chunks = max_chunks;
     c->page_stride = stride;
     c->step_batch = batch;
     c->step_entries = (int32_t)entries;
@@ -828,7 +832,8 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
     if (c->step_split) {
-        KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->num_sms, p, static_cast<cudaStream_t>(stream)));
+        KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->step_max_chunks, c->num_sms, p,
+                              static_cast<cudaStream_t>(stream)));
         ++c->launches;
     }
     if (fused) ++c->fused_launches;
@@ -912,6 +917,7 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     c->step_active = true;
     c->step_dev = true;
     c->step_split = true;   // the row split is only known on the device: always run the merge pass
+    c->step_max_chunks = row_chunks(c->cfg.max_pages_per_seq, c->dev_item_pages);
     c->step_batch = batch;
     c->step_entries = c->dev_entries_cap;
     c->page_stride = c->dev_stride;

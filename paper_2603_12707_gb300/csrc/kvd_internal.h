@@ -212,7 +212,8 @@ cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v);
 // Second pass: log-sum-exp merge of the partials of every split row, one warp
 // per (row, query head).  pdl: launched with programmatic dependent launch
 // (it lets the next kernel start at once and waits for the split pass).
-cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st);
+// max_chunks: an upper bound on the items of any row of the step (<= kMaxChunks).
+cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, const DecodeParams& p, cudaStream_t st);
 // fused: the append + attention kernel, launched with programmatic dependent
 // launch (it streams its first pages before the previous kernel finishes and
 // reads q / k_new / v_new and writes anything only after it has).

@@ -23,10 +23,12 @@ namespace {
 // before the first use, so a unit costs one round trip to L2.
 constexpr int kMergeSplit = 1;   // warps per (row, query head)
 constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
-constexpr int kMergeBatch = 32;  // items whose o is loaded before the first use
 constexpr int kMergeGridPerSm = 32;   // merge CTAs per SM at most (one-warp CTAs)
 
-template <int D>
+// BATCH: items whose o is loaded before the first use (registers: BATCH * D / 32
+// floats per lane); the launch picks the smallest BATCH that covers the step's
+// items per row, so a unit is one round trip and the CTAs stay small.
+template <int D, int BATCH>
 __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int b, int g, int hh, int part,
                                            int lane)
 {
@@ -37,10 +39,10 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
     float2 ml = make_float2(-INFINITY, 0.f);
     if (lane < nch) ml = __ldcg(&p.part_ml[slot(lane)]);
     const int d0 = part * (D / kMergeSplit) + lane * PER;
-    float vals[kMergeBatch][PER];
+    float vals[BATCH][PER];
     auto load = [&](int c0) {
 #pragma unroll
-    for (int u = 0; u < kMergeBatch; ++u) {
+    for (int u = 0; u < BATCH; ++u) {
         const int c = c0 + u;
         const float* src = p.part_o + slot(c < nch ? c : 0) * D + d0;
         if (c < nch) {
@@ -71,10 +73,10 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
     float acc[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) acc[j] = 0.f;
-    for (int c0 = 0; c0 < nch; c0 += kMergeBatch) {
+    for (int c0 = 0; c0 < nch; c0 += BATCH) {
         if (c0) load(c0);
 #pragma unroll
-        for (int u = 0; u < kMergeBatch; ++u) {
+        for (int u = 0; u < BATCH; ++u) {
             const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
 #pragma unroll
             for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[u][j], acc[j]);
@@ -94,7 +96,7 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
 // row descriptors come from the step's plan, not from the split pass, so a
 // warp reads its first one before waiting for the split pass: after the
 // wait only the partials are fetched.
-template <int D>
+template <int D, int BATCH>
 __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodeParams p, int pdl)
 {
     const int lane = threadIdx.x & 31;
@@ -113,7 +115,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
         if (!first) row = p.rows[b];
         if (row.y <= 1) continue;
         const int g = h / p.G;
-        merge_unit<D>(p, row, b, g, h - g * p.G, part, lane);
+        merge_unit<D, BATCH>(p, row, b, g, h - g * p.G, part, lane);
     }
 }
 
@@ -122,17 +124,26 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
 // The merge pass uses no shared memory; asking for the largest shared-memory
 // carveout keeps an SM that hosts its CTAs in the configuration of the split
 // pass, so the next layer's split-pass CTAs can still be placed there.
-template <int D>
-cudaError_t prepare_merge()
+template <int D, int BATCH>
+cudaError_t launch_merge_variant(const cudaLaunchConfig_t& cfg, const DecodeParams& p, int flag)
 {
     static cudaError_t status =
-        cudaFuncSetAttribute(merge_kernel<D>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    return status;
+        cudaFuncSetAttribute(merge_kernel<D, BATCH>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (status != cudaSuccess) return status;
+    return cudaLaunchKernelEx(&cfg, merge_kernel<D, BATCH>, p, flag);
 }
 
-cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cudaStream_t st)
+template <int D>
+cudaError_t launch_merge_d(int max_chunks, const cudaLaunchConfig_t& cfg, const DecodeParams& p, int flag)
 {
-    if (cudaError_t e = D == 128 ? prepare_merge<128>() : prepare_merge<64>()) return e;
+    if (max_chunks <= 4) return launch_merge_variant<D, 4>(cfg, p, flag);
+    if (max_chunks <= 8) return launch_merge_variant<D, 8>(cfg, p, flag);
+    if (max_chunks <= 16) return launch_merge_variant<D, 16>(cfg, p, flag);
+    return launch_merge_variant<D, 32>(cfg, p, flag);
+}
+
+cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, const DecodeParams& p, cudaStream_t st)
+{
     const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
                                                                    (int64_t)num_sms * kMergeGridPerSm));
@@ -147,8 +158,8 @@ cudaError_t launch_merge(int D, bool pdl, int num_sms, const DecodeParams& p, cu
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
     const int flag = pdl ? 1 : 0;
-    if (D == 128) return cudaLaunchKernelEx(&cfg, merge_kernel<128>, p, flag);
-    if (D == 64) return cudaLaunchKernelEx(&cfg, merge_kernel<64>, p, flag);
+    if (D == 128) return launch_merge_d<128>(max_chunks, cfg, p, flag);
+    if (D == 64) return launch_merge_d<64>(max_chunks, cfg, p, flag);
     return cudaErrorInvalidValue;
 }
 

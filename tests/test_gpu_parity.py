@@ -97,6 +97,29 @@ SMALL = [
 ]
 
 
+@pytest.mark.parametrize("max_items", [2, 3, 7, 12, 20, 32])
+@pytest.mark.parametrize("Hq,Hkv,d", [(8, 8, 128), (28, 4, 128), (14, 2, 64)])
+def test_merge_batch_variants(Hq, Hkv, d, max_items):
+    """The merge pass is compiled for 4, 8, 16 or 32 items in flight and the
+    launch picks the smallest that covers the step's longest row: one-page
+    items and a longest row of max_items pages exercise each variant, with
+    shorter rows (one item, several items) beside it."""
+    lens = [16 * max_items - 1, 40, 5, 16 * max(1, max_items // 2)]
+    cfg = wl.custom(f"merge{max_items}", 1, Hq, Hkv, d, len(lens), lens=lens, seed=400 + max_items,
+                    page_order="shuffled")
+    t = Tracked(cfg, extra_tokens=4, split_pages=1)
+    for _ in range(2):
+        t.begin_step()
+        for fused in (False, True):
+            out, q, _, _ = t.run_layer(0, fused=fused)
+            torch.cuda.synchronize()
+            ref, vmax = t.oracle(0, q)
+            assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv, what=(max_items, fused))
+            if not fused:
+                t.begin_step()
+    t.close()
+
+
 @pytest.mark.parametrize("split", [0, 1, 3, 64, 1024])
 @pytest.mark.parametrize("name,Hq,Hkv,d,lens", SMALL)
 def test_decode_matches_oracle_small(name, Hq, Hkv, d, lens, split):
