@@ -180,11 +180,13 @@ int push_updates(kv_cache* c, const std::vector<int32_t>& idx, const std::vector
 int32_t auto_item_pages(const kv_cache* c, int64_t total_units)
 {
     // About three work items per resident warp keeps the tail of the
-    // persistent schedule short; items stay within [2, 128] pages (long rows
-    // get larger items through the per-row cap on the number of items).
+    // persistent schedule short; a GQA item leaves a partial for each of its
+    // G query heads, so GQA aims at two.  Items stay within [2, 128] pages
+    // (long rows get larger items through the per-row cap on items).
     const int64_t warps = (int64_t)std::max(1, c->num_sms) * std::max(1, c->variant.ctas_per_sm) *
                           std::max(1, c->variant.warps);
-    const int64_t T = (total_units + 3 * warps - 1) / (3 * warps);
+    const int64_t per_warp = c->group > 1 ? 2 : 3;
+    const int64_t T = (total_units + per_warp * warps - 1) / (per_warp * warps);
     return (int32_t)std::min<int64_t>(128, std::max<int64_t>(2, T));
 }
 
