@@ -23,7 +23,11 @@ namespace {
 // before the first use, so a unit costs one round trip to L2.
 constexpr int kMergeSplit = 1;   // warps per (row, query head)
 constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
-constexpr int kMergeGridPerSm = 32;   // merge CTAs per SM at most (one-warp CTAs)
+// Merge CTAs per SM at most.  The whole merge grid must fit beside the
+// resident split pass (8 one-warp CTAs per SM): a merge CTA that waits for a
+// slot holds back the next layer, which may start only once every merge CTA
+// has started.  Rows with more units than the grid loop over them.
+constexpr int kMergeGridPerSm = 16;
 
 // BATCH: items whose o is loaded before the first use (registers: BATCH * D / 32
 // floats per lane); the launch picks the smallest BATCH that covers the step's
