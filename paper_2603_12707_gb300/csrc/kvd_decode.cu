@@ -523,6 +523,11 @@ cudaError_t variant_info(DecodeVariant* v)
     if (e != cudaSuccess) return e;
     v->warps = kWarps;
     v->smem_bytes = Geo<D, GQA>::kSmem;
+    cudaFuncAttributes a0, a1;
+    e = cudaFuncGetAttributes(&a0, decode_kernel<D, GQA, false>);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&a1, decode_kernel<D, GQA, true>);
+    if (e != cudaSuccess) return e;
+    v->regs = std::max(a0.numRegs, a1.numRegs);
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v->ctas_per_sm, decode_kernel<D, GQA, false>, kWarps * 32,
                                                          Geo<D, GQA>::kSmem);
 }

@@ -834,7 +834,11 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
     if (c->step_split) {
-        KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->step_max_chunks, c->num_sms, p,
+        // Launched early (fused), the merge CTAs sit beside the resident split pass.
+        const int split_regs =
+            fused ? ((c->variant.ctas_per_sm * c->variant.warps + 3) / 4) * warp_register_allocation(c->variant.regs)
+                  : 0;
+        KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->step_max_chunks, c->num_sms, split_regs, p,
                               static_cast<cudaStream_t>(stream)));
         ++c->launches;
     }

@@ -207,13 +207,22 @@ struct DecodeVariant {
     int warps;        // warps per CTA
     int smem_bytes;   // dynamic shared memory per CTA
     int ctas_per_sm;  // occupancy at that shared memory
+    int regs;         // registers per thread (the larger of the two variants)
 };
+
+// Registers one warp is allocated for `regs` registers per thread (per-thread
+// counts are allocated in multiples of 8).
+inline int warp_register_allocation(int regs) { return ((regs + 7) / 8) * 8 * 32; }
+constexpr int kRegistersPerSubpartition = 16384;   // an SM's 64 K registers over its 4 schedulers
 cudaError_t decode_variant_info(int D, bool gqa, DecodeVariant* v);
 // Second pass: log-sum-exp merge of the partials of every split row, one warp
 // per (row, query head).  pdl: launched with programmatic dependent launch
 // (it lets the next kernel start at once and waits for the split pass).
 // max_chunks: an upper bound on the items of any row of the step (<= kMaxChunks).
-cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, const DecodeParams& p, cudaStream_t st);
+// split_regs_per_subpartition: registers the resident split pass holds on
+// each of an SM's four schedulers (0: nothing resident beside it).
+cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, int split_regs_per_subpartition,
+                         const DecodeParams& p, cudaStream_t st);
 // fused: the append + attention kernel, launched with programmatic dependent
 // launch (it streams its first pages before the previous kernel finishes and
 // reads q / k_new / v_new and writes anything only after it has).

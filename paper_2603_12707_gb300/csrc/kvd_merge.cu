@@ -123,8 +123,6 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
     }
 }
 
-}  // namespace
-
 // The merge pass uses no shared memory; asking for the largest shared-memory
 // carveout keeps an SM that hosts its CTAs in the configuration of the split
 // pass, so the next layer's split-pass CTAs can still be placed there.
@@ -137,20 +135,56 @@ cudaError_t launch_merge_variant(const cudaLaunchConfig_t& cfg, const DecodePara
     return cudaLaunchKernelEx(&cfg, merge_kernel<D, BATCH>, p, flag);
 }
 
-template <int D>
-cudaError_t launch_merge_d(int max_chunks, const cudaLaunchConfig_t& cfg, const DecodeParams& p, int flag)
+template <int D, int BATCH>
+int merge_registers()
 {
-    if (max_chunks <= 4) return launch_merge_variant<D, 4>(cfg, p, flag);
-    if (max_chunks <= 8) return launch_merge_variant<D, 8>(cfg, p, flag);
-    if (max_chunks <= 16) return launch_merge_variant<D, 16>(cfg, p, flag);
+    static int regs = [] {
+        cudaFuncAttributes a;
+        return cudaFuncGetAttributes(&a, merge_kernel<D, BATCH>) == cudaSuccess ? a.numRegs : 255;
+    }();
+    return regs;
+}
+
+template <int D>
+int merge_registers(int batch)
+{
+    return batch == 4 ? merge_registers<D, 4>() : batch == 8 ? merge_registers<D, 8>()
+         : batch == 16 ? merge_registers<D, 16>() : merge_registers<D, 32>();
+}
+
+template <int D>
+cudaError_t launch_merge_d(int batch, cudaLaunchConfig_t& cfg, const DecodeParams& p, int flag)
+{
+    if (batch == 4) return launch_merge_variant<D, 4>(cfg, p, flag);
+    if (batch == 8) return launch_merge_variant<D, 8>(cfg, p, flag);
+    if (batch == 16) return launch_merge_variant<D, 16>(cfg, p, flag);
     return launch_merge_variant<D, 32>(cfg, p, flag);
 }
 
-cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, const DecodeParams& p, cudaStream_t st)
+}  // namespace
+
+// The smallest variant whose items in flight cover the step's longest row,
+// unless its registers would leave part of the grid waiting for a slot beside
+// the resident split pass: then fewer items in flight (a second round trip
+// for the longest rows only) with fewer registers.
+cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, int split_regs_per_subpartition,
+                         const DecodeParams& p, cudaStream_t st)
 {
-    const int64_t warps = (int64_t)p.batch * p.H_q * kMergeSplit;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((warps + kMergeWarps - 1) / kMergeWarps,
-                                                                   (int64_t)num_sms * kMergeGridPerSm));
+    const int64_t units = (int64_t)p.batch * p.H_q * kMergeSplit;
+    const int64_t want = std::max<int64_t>(1, std::min<int64_t>((units + kMergeWarps - 1) / kMergeWarps,
+                                                                  (int64_t)num_sms * kMergeGridPerSm));
+    int batch = max_chunks <= 4 ? 4 : max_chunks <= 8 ? 8 : max_chunks <= 16 ? 16 : 32;
+    int64_t grid = want;
+    for (;; batch /= 2) {
+        const int regs = D == 128 ? merge_registers<128>(batch) : merge_registers<64>(batch);
+        const int64_t per_sub = (kRegistersPerSubpartition - split_regs_per_subpartition) /
+                                (warp_register_allocation(regs) * kMergeWarps);
+        const int64_t fit = (int64_t)num_sms * std::min<int64_t>(kMergeGridPerSm, 4 * per_sub);
+        if (fit >= want || batch == 4) {
+            grid = std::max<int64_t>(1, std::min(want, fit));
+            break;
+        }
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(kMergeWarps * 32);
@@ -162,8 +196,8 @@ cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, const Dec
     cfg.attrs = attr;
     cfg.numAttrs = pdl ? 1 : 0;
     const int flag = pdl ? 1 : 0;
-    if (D == 128) return launch_merge_d<128>(max_chunks, cfg, p, flag);
-    if (D == 64) return launch_merge_d<64>(max_chunks, cfg, p, flag);
+    if (D == 128) return launch_merge_d<128>(batch, cfg, p, flag);
+    if (D == 64) return launch_merge_d<64>(batch, cfg, p, flag);
     return cudaErrorInvalidValue;
 }
 
