@@ -138,17 +138,23 @@ def gpu_smi_id(torch, dev):
 
 
 # --------------------------------------------------------- kernel traffic
-def kernel_code_hash(path):
-    """sha256 (16 hex digits) of a source file's code: line comments, blank
-    lines and surrounding whitespace removed, so a comment edit keeps a
-    capture valid and any code edit voids it."""
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2603_12707_gb300", "csrc", f)
+                  for f in ("kvd_decode_kernel.cuh", "kvd_ptx.cuh")]
+
+
+def kernel_code_hash(paths):
+    """sha256 (16 hex digits) of the split-pass kernel's device code: line
+    comments, blank lines and surrounding whitespace removed, so a comment
+    edit keeps a capture valid and any code edit voids it."""
     import re
-    with open(path) as f:
-        lines = [re.sub(r"//.*$", "", l).strip() for l in f]
+    lines = []
+    for path in paths:
+        with open(path) as f:
+            lines += [re.sub(r"//.*$", "", l).strip() for l in f]
     return hashlib.sha256("\n".join(l for l in lines if l).encode()).hexdigest()[:16]
 
 
-def committed_traffic(kernel_src, workload, algorithmic_bytes):
+def committed_traffic(kernel_srcs, workload, algorithmic_bytes):
     """DRAM bytes per launch of the decode kernel: the committed ncu capture's
     traffic / algorithmic ratio for this workload times this launch's
     algorithmic bytes; None unless the capture was taken on the current
@@ -158,7 +164,7 @@ def committed_traffic(kernel_src, workload, algorithmic_bytes):
         return None
     with open(p) as f:
         d = json.load(f)
-    h = kernel_code_hash(kernel_src)
+    h = kernel_code_hash(kernel_srcs)
     cap = d.get("captures", {}).get(workload)
     if d.get("source_sha256_16") != h or cap is None:
         return None
@@ -560,8 +566,7 @@ def main():
     attn_bytes = statistics.mean(r["attn_bytes"])
     peak, peak_kind = measured_peaks()
     achieved = attn_bytes / (attn_ms / 1e3) / 1e9
-    traffic = None if args.unfused else committed_traffic(
-        os.path.join(ROOT, "paper_2603_12707_gb300", "csrc", "kvd_decode.cu"), cfg.name, attn_bytes)
+    traffic = None if args.unfused else committed_traffic(KERNEL_SOURCES, cfg.name, attn_bytes)
     out = {
         "metric": METRIC, "value": round(gbs, 2), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
