@@ -223,11 +223,22 @@ def run_gpu(args, rank, world):
                              split_pages=args.split_pages)
         sess.fill_prefix()
         L, B = cfg.num_layers, cfg.batch
+        # Every layer's q, k_new, v_new live in one device buffer and every
+        # layer's output in another, so the end-to-end leg moves a step's
+        # inputs and outputs in one copy each way.
+        Hq, Hkv, d = cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
+        per_layer = B * (Hq + 2 * Hkv) * d
+        d_in = torch.empty(L * per_layer, dtype=torch.bfloat16, device="cuda")
+        d_out = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device="cuda")
         qs, ks, vs = [], [], []
         for l in range(L):
+            x = d_in[l * per_layer:(l + 1) * per_layer]
+            qs.append(x[:B * Hq * d].view(B, Hq, d))
+            ks.append(x[B * Hq * d:B * (Hq + Hkv) * d].view(B, Hkv, d))
+            vs.append(x[B * (Hq + Hkv) * d:].view(B, Hkv, d))
             q, k, v = wl.step_inputs(cfg, 0, l, "cuda")
-            qs.append(q), ks.append(k), vs.append(v)
-        outs = [torch.empty_like(q) for q in qs]
+            qs[l].copy_(q), ks[l].copy_(k), vs[l].copy_(v)
+        outs = [d_out[l] for l in range(L)]
     stream.synchronize()
     log(f"[rank {rank}] setup {time.perf_counter() - t_setup:.1f} s; pool "
         f"{sess.query().pool_bytes / 2**30:.1f} GiB")
@@ -328,33 +339,22 @@ def run_gpu(args, rank, world):
     assert st.device_error == 0, st.device_error
     # graph replays do not pass through the library: count the captured launches
     timed_launches = graphs[2] * args.steps if graphs is not None else st.kernel_launches - launches0
-    if graphs is not None:
-        kd.kv_cache_device_steps(sess.h, B, False, stream)   # host-driven steps from here on
 
-    # ---- end to end: host inputs -> device -> host outputs, every step.
-    # A step's q, k_new, v_new of all layers sit in one pinned host buffer
-    # and go over in one copy; all layers' outputs come back in one copy.
+    # ---- end to end: host inputs -> device -> host outputs, every step: a
+    # step's q, k_new, v_new of all layers go over from pinned host memory in
+    # one copy, the step runs as timed above (graph replay, or the host calls
+    # with --host-steps / --unfused) and all layers' outputs come back in one
+    # copy.
     e2e = None
     if not args.no_e2e:
-        Hq, Hkv, d = cfg.num_q_heads, cfg.num_kv_heads, cfg.head_dim
-        per_layer = B * (Hq + 2 * Hkv) * d
-        h_in = torch.empty(L * per_layer, dtype=torch.bfloat16).pin_memory()
-        for l in range(L):
-            h_in[l * per_layer:(l + 1) * per_layer] = torch.cat(
-                [qs[l].reshape(-1), ks[l].reshape(-1), vs[l].reshape(-1)]).cpu()
-        d_in = torch.empty_like(h_in, device="cuda")
-        d_out = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device="cuda")
+        h_in = d_in.cpu().pin_memory()
         h_out = torch.empty_like(d_out, device="cpu").pin_memory()
-
-        def views(l):
-            x = d_in[l * per_layer:(l + 1) * per_layer]
-            return (x[:B * Hq * d].view(B, Hq, d), x[B * Hq * d:B * (Hq + Hkv) * d].view(B, Hkv, d),
-                    x[B * (Hq + Hkv) * d:].view(B, Hkv, d))
-
         e_bytes = 0
         h2d = h_in.numel() * 2
         d2h = h_out.numel() * 2
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        # (device steps stay enabled from the capture on: re-enabling them
+        # could move the scratch buffers the captured graphs point at)
         torch.cuda.synchronize()
         if world > 1:
             torch.distributed.barrier()
@@ -366,14 +366,7 @@ def run_gpu(args, rank, world):
                 a, p = layer_bytes(cfg, att)
                 e_bytes += L * (a + p)
                 d_in.copy_(h_in, non_blocking=True)
-                sess.begin_step()
-                for l in range(L):
-                    q, k, v = views(l)
-                    if args.unfused:
-                        sess.append(l, k, v)
-                        sess.attend(l, q, d_out[l])
-                    else:
-                        sess.append_attend(l, q, k, v, d_out[l])
+                step()
                 h_out.copy_(d_out, non_blocking=True)
             s1.record(stream)
         stream.synchronize()
