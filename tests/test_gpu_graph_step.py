@@ -136,3 +136,49 @@ def test_device_step_reports_an_exhausted_pool(kvlib):
     for i, s_ in enumerate(seqs):
         assert kd.kv_seq_info(h, s_)[1] == m.pages[i]
     kd.kv_cache_destroy(h)
+
+
+def test_device_steps_interleaved_with_host_lifecycle(kvlib):
+    """Device-side steps mixed with host-side lifecycle calls (free a
+    sequence, create one, reserve its prompt) on a shuffled pool: after every
+    phase each live sequence holds the length and the pages the allocator
+    model hands out for the same calls, and the free count agrees."""
+    num_pages, P = 40, 16
+    cfg = kd.make_config(1, 8, 8, 64, num_pages, 6, 8)
+    h = kd.kv_cache_create(cfg)
+    perm = np.random.default_rng(17).permutation(num_pages)
+    kd.kv_cache_set_page_order(h, perm)
+    m = PagePoolModel(num_pages, P, 6, 8)
+    m.set_page_order(perm)
+    batch = []
+    for n in (5, 16, 30, 47):
+        s_ = kd.kv_seq_create(h)
+        assert s_ == m.seq_create()
+        kd.kv_seq_reserve(h, s_, n)
+        m.seq_reserve(s_, n)
+        batch.append(s_)
+    kd.kv_cache_device_steps(h, 6)
+
+    def check():
+        st = kd.kv_cache_query(h)
+        assert st.free_pages == len(m.free) and st.pages_in_use == num_pages - len(m.free)
+        for s_ in batch:
+            assert kd.kv_seq_info(h, s_) == (m.lens[s_], m.pages[s_]), s_
+
+    for phase in range(3):
+        ids = torch.tensor(batch, dtype=torch.int32, device="cuda")
+        for _ in range(7):
+            kd.kv_begin_step_device(h, len(batch), ids)
+            m.begin_step(batch)
+        torch.cuda.synchronize()
+        check()
+        victim = batch[(phase + 1) % len(batch)]
+        kd.kv_seq_free(h, victim)
+        m.seq_free(victim)
+        new = kd.kv_seq_create(h)
+        assert new == m.seq_create()
+        kd.kv_seq_reserve(h, new, 20)
+        m.seq_reserve(new, 20)
+        batch[batch.index(victim)] = new
+        check()
+    kd.kv_cache_destroy(h)
