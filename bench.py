@@ -308,6 +308,7 @@ def run_gpu(args, rank, world):
     attended_per_step = []
     n_ev = 2 * L if args.unfused else 2
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
+    step_ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
@@ -316,15 +317,18 @@ def run_gpu(args, rank, world):
     with ClockSampler(gpu_smi_id(torch, dev)) as clocks:
         with torch.cuda.stream(stream):
             start.record(stream)
+            step_ev[0].record(stream)
             for s in range(args.steps):
                 attended_per_step.append([int(n) + 1 for n in sess.lens])
                 step(ev[s])
+                step_ev[s + 1].record(stream)
             stop.record(stream)
         stream.synchronize()
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     ms = start.elapsed_time(stop)
+    step_ms = [step_ev[i].elapsed_time(step_ev[i + 1]) for i in range(args.steps)]
     if args.unfused:
         attn_ms = [evs[2 * l].elapsed_time(evs[2 * l + 1]) for evs in ev for l in range(L)]
     else:
@@ -377,7 +381,7 @@ def run_gpu(args, rank, world):
         assert st.device_error == 0
 
     sess.close()
-    return {"ms": ms, "attn_ms": attn_ms, "step_bytes": step_bytes, "attn_bytes": attn_bytes,
+    return {"ms": ms, "step_ms": step_ms, "attn_ms": attn_ms, "step_bytes": step_bytes, "attn_bytes": attn_bytes,
             "launches": timed_launches,
             "clocks": clocks.summary(), "e2e": e2e, "cfg": cfg, "L": L}
 
@@ -569,6 +573,8 @@ def main():
                    "step_driver": "cuda_graph" if args.graph else "host",
                    "parallelism": f"replicas x{world}"},
         "steps_per_s": round(steps_per_s * 1.0, 3),
+        "step_ms_median": round(statistics.median(r["step_ms"]), 4),
+        "step_ms_min": round(min(r["step_ms"]), 4),
         "pct_of_measured_hbm": round(100 * gbs / world / peak, 2),
         "pct_of_nominal_8tbs": round(100 * gbs / world / NOMINAL_HBM_GBS, 2),
         "roofline": {"bound": "hbm", "kernel": "decode_attention" if args.unfused else "decode_attention_append",
