@@ -676,12 +676,20 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         total_units += (int64_t)np_after[b] * c->cfg.num_kv_heads;
     }
     const int32_t T = c->split_override ? c->split_override : auto_item_pages(c, total_units);
+    // Plan order: longest rows first (stable), when the batch fits one launch.
+    const bool use_order = batch <= kPatchMax;
+    std::vector<int32_t> order((size_t)batch), rank((size_t)batch);
+    for (int32_t b = 0; b < batch; ++b) order[b] = b;
+    if (use_order)
+        std::stable_sort(order.begin(), order.end(),
+                         [&](int32_t x, int32_t y) { return np_after[x] > np_after[y]; });
+    for (int32_t i = 0; i < batch; ++i) rank[order[i]] = i;
     int64_t entries = 0;
     int32_t stride = 1;
     bool split = false;
     int32_t max_chunks = 1;
     for (int32_t b = 0; b < batch; ++b) {
-        const int nch = row_chunks(np_after[b], T);
+        const int nch = row_chunks(np_after[b], row_item_pages(T, rank[b], batch));
         entries += nch;
         split = split || nch > 1;
         max_chunks = std::max(max_chunks, nch);
@@ -717,12 +725,9 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         pa.rows = c->rows;
         pa.err = c->err;
         // Longest rows first: their items start early and the tail is short.
-        pa.use_order = batch <= kPatchMax ? 1 : 0;
-        if (pa.use_order) {
-            for (int32_t b = 0; b < batch; ++b) pa.order[b] = b;
-            std::stable_sort(pa.order, pa.order + batch,
-                             [&](int32_t x, int32_t y) { return np_after[x] > np_after[y]; });
-        }
+        pa.use_order = use_order ? 1 : 0;
+        if (use_order)
+            for (int32_t i = 0; i < batch; ++i) pa.order[i] = order[i];
         for (int32_t b0 = 0; b0 < batch; b0 += kPatchMax) {
             const int32_t n = std::min(kPatchMax, batch - b0);
             patch.n = n;
@@ -923,7 +928,7 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     c->step_active = true;
     c->step_dev = true;
     c->step_split = true;   // the row split is only known on the device: always run the merge pass
-    c->step_max_chunks = row_chunks(c->cfg.max_pages_per_seq, c->dev_item_pages);
+    c->step_max_chunks = row_chunks(c->cfg.max_pages_per_seq, row_item_pages(c->dev_item_pages, batch, batch));
     c->step_batch = batch;
     c->step_entries = c->dev_entries_cap;
     c->page_stride = c->dev_stride;

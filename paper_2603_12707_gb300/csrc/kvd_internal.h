@@ -30,6 +30,16 @@ struct PlanEntry {
     int32_t slot_base;  // first partial slot of the row; slot = (slot_base + chunk) * H_kv + g
 };
 
+// Target item size of the row planned at position i of n (rows are planned
+// longest first): the last rows get smaller items, so a launch ends on short
+// items and the warps run out of work at nearly the same time.
+__host__ __device__ inline int row_item_pages(int T, int i, int n)
+{
+    if (10 * (int64_t)i >= 9 * (int64_t)n) return T >= 4 ? T / 4 : 1;
+    if (10 * (int64_t)i >= 7 * (int64_t)n) return T >= 2 ? T / 2 : 1;
+    return T;
+}
+
 // Split policy shared by host and device.  A row of np pages is cut into
 // nch items of near-equal size: the target size T, raised for long rows so a
 // row never has more than kMaxChunks items (which bounds the merge).
