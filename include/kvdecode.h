@@ -249,7 +249,11 @@ KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batc
  * allocator's view is refreshed from the device (a device synchronisation)
  * by the next call that needs it: kv_seq_reserve, kv_seq_free, kv_seq_info,
  * kv_begin_step, kv_cache_query, kv_write_tokens, kv_read_tokens,
- * kv_cache_set_page_order, or kv_cache_sync. */
+ * kv_cache_set_page_order, or kv_cache_sync.  Graphs captured while device
+ * steps are enabled stay valid until they are disabled, enabled again (which
+ * may resize the buffers) or the cache is destroyed: meanwhile a host-planned
+ * step that would need larger buffers fails with KVC_ERR_INVALID instead of
+ * moving them. */
 KVC_API int kv_cache_device_steps(kv_cache *cache, int32_t max_batch, int32_t enable, void *stream);
 
 /* kv_begin_step with everything on the device: seq_ids is DEVICE memory

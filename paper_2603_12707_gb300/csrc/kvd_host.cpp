@@ -192,6 +192,12 @@ int32_t auto_item_pages(const kv_cache* c, int64_t total_units)
 
 int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, int64_t page_ids, cudaStream_t st)
 {
+    // While device steps are enabled, captured graphs may hold these buffers'
+    // addresses: they must not move.
+    if (c->dev_mode && (page_ids > c->item_pages_cap || entries > c->plan_cap || slots > c->slot_cap))
+        return fail(KVC_ERR_INVALID,
+                    "the step needs larger plan buffers than kv_cache_device_steps reserved, and graphs "
+                    "captured since may use them: disable device steps first");
     if (page_ids > c->item_pages_cap) {
         const int64_t cap = std::max<int64_t>(page_ids, c->item_pages_cap + c->item_pages_cap / 2);
         if (c->item_pages) KVD_CUDA(cudaFreeAsync(c->item_pages, st));
@@ -879,6 +885,7 @@ int kv_cache_device_steps(kv_cache* c, int32_t max_batch, int32_t enable, void* 
     }
     if (max_batch < 1 || max_batch > c->cfg.max_seqs)
         return fail(KVC_ERR_INVALID, "kv_cache_device_steps: max_batch outside 1 .. max_seqs");
+    c->dev_mode = false;   // (re-)enabling may resize the buffers
     // Work-item size from the pages now held (steps add a token per sequence).
     const int32_t T = c->split_override
                           ? c->split_override

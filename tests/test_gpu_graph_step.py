@@ -182,3 +182,25 @@ def test_device_steps_interleaved_with_host_lifecycle(kvlib):
         batch[batch.index(victim)] = new
         check()
     kd.kv_cache_destroy(h)
+
+
+def test_host_step_cannot_move_buffers_under_device_steps(kvlib):
+    """Device steps reserve plan buffers (captured graphs point at them); a
+    host-planned step that needs more fails with KVC_ERR_INVALID and changes
+    nothing, and works once device steps are disabled."""
+    cfg = kd.make_config(1, 8, 8, 64, 600, 4, 128)
+    h = kd.kv_cache_create(cfg)
+    seqs = [kd.kv_seq_create(h) for _ in range(4)]
+    for s_ in seqs:
+        kd.kv_seq_reserve(h, s_, 1900)
+    kd.kv_cache_set_split_pages(h, 4)
+    kd.kv_cache_device_steps(h, 2)          # room for 2 rows x 32 items
+    before = [kd.kv_seq_info(h, s_) for s_ in seqs]
+    with pytest.raises(kd.KVDecodeError) as ei:
+        kd.kv_begin_step(h, seqs)           # 4 rows x 30 items
+    assert ei.value.code == kd.KVC_ERR_INVALID and "disable device steps" in str(ei.value)
+    assert [kd.kv_seq_info(h, s_) for s_ in seqs] == before
+    kd.kv_cache_device_steps(h, 2, False)
+    kd.kv_begin_step(h, seqs)
+    assert [kd.kv_seq_info(h, s_)[0] for s_ in seqs] == [1901] * 4
+    kd.kv_cache_destroy(h)
