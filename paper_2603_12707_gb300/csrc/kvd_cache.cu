@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(1024)
                 len = 1;
             }
             np = (len + kPageSize - 1) / kPageSize;
-            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch));
+            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch), a.chunk_cap);
         }
         int total;
         const int off = carry + block_exclusive_scan(nch, &total);
@@ -168,7 +168,7 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
             seq = a.step_seq[b];
             len = max(1, a.seq_len[seq]);
             np = (len + kPageSize - 1) / kPageSize;
-            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch));
+            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch), a.chunk_cap);
         }
         int total;
         const int off = carry + block_exclusive_scan(nch, &total);

@@ -118,6 +118,7 @@ struct kv_cache {
     int32_t dev_item_pages = 0;
     int32_t dev_entries_cap = 0;
     int32_t dev_stride = 0;
+    int32_t dev_chunk_cap = kChunkCap;
     int32_t* d_free = nullptr;                  // [num_pages]
     int32_t* d_small = nullptr;                 // [0] free top, [1] plan entries of the step
 
@@ -188,6 +189,17 @@ int32_t auto_item_pages(const kv_cache* c, int64_t total_units)
     const int64_t per_warp = c->group > 1 ? 2 : 3;
     const int64_t T = (total_units + per_warp * warps - 1) / (per_warp * warps);
     return (int32_t)std::min<int64_t>(128, std::max<int64_t>(2, T));
+}
+
+// Items per row at most: the usual cap, or twice it when rows x KV heads x
+// the usual cap would leave resident warps without an item and some row
+// (of up to max_pages pages) is long enough to use more items of T pages.
+int32_t chunk_cap(const kv_cache* c, int64_t rows, int64_t max_pages, int32_t T)
+{
+    const int64_t warps = (int64_t)std::max(1, c->num_sms) * std::max(1, c->variant.ctas_per_sm) *
+                          std::max(1, c->variant.warps);
+    const bool few_units = rows * c->cfg.num_kv_heads * kChunkCap < warps;
+    return few_units && max_pages > (int64_t)kChunkCap * T ? kMaxChunks : kChunkCap;
 }
 
 int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, int64_t page_ids, cudaStream_t st)
@@ -690,12 +702,13 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         std::stable_sort(order.begin(), order.end(),
                          [&](int32_t x, int32_t y) { return np_after[x] > np_after[y]; });
     for (int32_t i = 0; i < batch; ++i) rank[order[i]] = i;
+    const int32_t cap = chunk_cap(c, batch, *std::max_element(np_after.begin(), np_after.end()), T);
     int64_t entries = 0;
     int32_t stride = 1;
     bool split = false;
     int32_t max_chunks = 1;
     for (int32_t b = 0; b < batch; ++b) {
-        const int nch = row_chunks(np_after[b], row_item_pages(T, rank[b], batch));
+        const int nch = row_chunks(np_after[b], row_item_pages(T, rank[b], batch), cap);
         entries += nch;
         split = split || nch > 1;
         max_chunks = std::max(max_chunks, nch);
@@ -729,6 +742,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         pa.page_table = c->page_table();
         pa.plan = c->plan;
         pa.rows = c->rows;
+        pa.chunk_cap = cap;
         pa.err = c->err;
         // Longest rows first: their items start early and the tail is short.
         pa.use_order = use_order ? 1 : 0;
@@ -890,8 +904,9 @@ int kv_cache_device_steps(kv_cache* c, int32_t max_batch, int32_t enable, void* 
     const int32_t T = c->split_override
                           ? c->split_override
                           : auto_item_pages(c, c->pages_in_use * (int64_t)c->cfg.num_kv_heads);
-    const int32_t entries = max_batch * kMaxChunks;
-    const int32_t stride = std::max(T, (c->cfg.max_pages_per_seq + kMaxChunks - 1) / kMaxChunks) + 1;
+    const int32_t cap = chunk_cap(c, max_batch, c->cfg.max_pages_per_seq, T);
+    const int32_t entries = max_batch * cap;
+    const int32_t stride = std::max(T, (c->cfg.max_pages_per_seq + cap - 1) / cap) + 1;
     if (int rc = grow_scratch(c, entries, (int64_t)entries * c->cfg.num_kv_heads, (int64_t)entries * stride, st))
         return rc;
     if (!c->d_free) KVD_CUDA(cudaMalloc((void**)&c->d_free, (size_t)c->cfg.num_pages * sizeof(int32_t)));
@@ -901,6 +916,7 @@ int kv_cache_device_steps(kv_cache* c, int32_t max_batch, int32_t enable, void* 
     c->dev_item_pages = T;
     c->dev_entries_cap = entries;
     c->dev_stride = stride;
+    c->dev_chunk_cap = cap;
     return push_free_stack(c, st);
 }
 
@@ -925,6 +941,7 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     a.plan = c->plan;
     a.rows = c->rows;
     a.n_entries = c->d_small + 1;
+    a.chunk_cap = c->dev_chunk_cap;
     a.err = c->err;
     KVD_CUDA(launch_step_device(a, st));
     ++c->launches;
@@ -935,7 +952,8 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     c->step_active = true;
     c->step_dev = true;
     c->step_split = true;   // the row split is only known on the device: always run the merge pass
-    c->step_max_chunks = row_chunks(c->cfg.max_pages_per_seq, row_item_pages(c->dev_item_pages, batch, batch));
+    c->step_max_chunks =
+        row_chunks(c->cfg.max_pages_per_seq, row_item_pages(c->dev_item_pages, batch, batch), c->dev_chunk_cap);
     c->step_batch = batch;
     c->step_entries = c->dev_entries_cap;
     c->page_stride = c->dev_stride;

@@ -10,7 +10,8 @@ namespace kvd {
 
 constexpr int kPageSize = 16;          // tokens per page (the only supported P)
 constexpr int kMaxGroup = 8;           // query heads per KV head handled by one MMA N-tile
-constexpr int kMaxChunks = 32;         // work items per (row, KV head) at most
+constexpr int kMaxChunks = 64;         // work items per (row, KV head) at most
+constexpr int kChunkCap = 32;          // the usual cap; 64 only when few rows must fill the GPU
 constexpr int kMaxItemPages = 1024;    // largest target item size a caller may request
 constexpr int kPatchMax = 1024;        // step entries carried in one launch's parameters
 constexpr int kScatterMax = 2048;      // int32 updates carried in one launch's parameters
@@ -42,10 +43,10 @@ __host__ __device__ inline int row_item_pages(int T, int i, int n)
 
 // Split policy shared by host and device.  A row of np pages is cut into
 // nch items of near-equal size: the target size T, raised for long rows so a
-// row never has more than kMaxChunks items (which bounds the merge).
-__host__ __device__ inline int row_chunks(int np, int T)
+// row never has more than `cap` items (which bounds the merge).
+__host__ __device__ inline int row_chunks(int np, int T, int cap = kChunkCap)
 {
-    const int t_row = (np + kMaxChunks - 1) / kMaxChunks;
+    const int t_row = (np + cap - 1) / cap;
     const int Tb = T > t_row ? T : t_row;
     return (np + Tb - 1) / Tb;
 }
@@ -79,6 +80,7 @@ struct PlanArgs {
     int32_t* page_table; // [max_seqs][max_pages]
     PlanEntry* plan;     // [n_entries]
     int2* rows;          // [batch]: (first partial slot, items) of each batch row
+    int32_t chunk_cap;   // items per row at most (kChunkCap or kMaxChunks)
     int32_t* err;
 };
 
@@ -97,6 +99,7 @@ struct StepDevArgs {
     PlanEntry* plan;
     int2* rows;
     int32_t* n_entries;       // out: plan entries of the step
+    int32_t chunk_cap;        // items per row at most (kChunkCap or kMaxChunks)
     int32_t* err;
 };
 

@@ -18,9 +18,10 @@ namespace {
 // Merge pass.  SPLIT warps merge a split row's items for one query head
 // h = g * G + hh of batch row b, each owning D / SPLIT dims:
 //     M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c,
-// lane c holding item c's (m, l) and every lane D / (32 * SPLIT) dims of o.
-// All loads (m, l and the o of every item, at most kMaxChunks) are issued
-// before the first use, so a unit costs one round trip to L2.
+// lane c holding the (m, l) of item c (and, in the 32-item variant, of item
+// c + 32: rows of up to 64 items) and every lane D / (32 * SPLIT) dims of o.  The loads of (m, l) and of the first BATCH items' o are
+// issued before the first use, so a row of up to BATCH items costs one round
+// trip to L2.
 constexpr int kMergeSplit = 1;   // warps per (row, query head)
 constexpr int kMergeWarps = 1;   // warps per CTA: small CTAs fit beside the split pass's
 // Merge CTAs per SM at most.  The whole merge grid must fit beside the
@@ -40,8 +41,13 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
     static_assert(PER == 1 || PER == 2 || PER == 4, "dims per lane");
     const int nch = row.y;
     auto slot = [&](int c) { return ((int64_t)(row.x + c) * p.H_kv + g) * p.G + hh; };
-    float2 ml = make_float2(-INFINITY, 0.f);
-    if (lane < nch) ml = __ldcg(&p.part_ml[slot(lane)]);
+    // Only the 32-item variant takes rows of more than 32 items; the smaller
+    // variants keep their registers (they must fit beside the split pass).
+    constexpr bool kTwoSlots = BATCH == 32;
+    float2 ml0 = make_float2(-INFINITY, 0.f), ml1 = make_float2(-INFINITY, 0.f);
+    if (lane < nch) ml0 = __ldcg(&p.part_ml[slot(lane)]);
+    if constexpr (kTwoSlots)
+        if (lane + 32 < nch) ml1 = __ldcg(&p.part_ml[slot(lane + 32)]);
     const int d0 = part * (D / kMergeSplit) + lane * PER;
     float vals[BATCH][PER];
     auto load = [&](int c0) {
@@ -66,14 +72,15 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
     }
     };
     load(0);
-    float M = ml.x;
+    float M = kTwoSlots ? fmaxf(ml0.x, ml1.x) : ml0.x;
 #pragma unroll
     for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float e = (lane < nch) ? ex2(ml.x - M) : 0.f;
-    float L = e * ml.y;
+    const float e0 = (lane < nch) ? ex2(ml0.x - M) : 0.f;
+    const float e1 = (kTwoSlots && lane + 32 < nch) ? ex2(ml1.x - M) : 0.f;
+    float L = kTwoSlots ? e0 * ml0.y + e1 * ml1.y : e0 * ml0.y;
 #pragma unroll
     for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    const float wgt = e / L;
+    const float w0 = e0 / L, w1 = e1 / L;   // weights of items lane and lane + 32
     float acc[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) acc[j] = 0.f;
@@ -81,7 +88,7 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
         if (c0) load(c0);
 #pragma unroll
         for (int u = 0; u < BATCH; ++u) {
-            const float wc = __shfl_sync(0xffffffffu, wgt, (c0 + u) & 31);
+            const float wc = __shfl_sync(0xffffffffu, (!kTwoSlots || c0 + u < 32) ? w0 : w1, (c0 + u) & 31);
 #pragma unroll
             for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[u][j], acc[j]);
         }
@@ -175,12 +182,14 @@ cudaError_t launch_merge(int D, bool pdl, int max_chunks, int num_sms, int split
                                                                   (int64_t)num_sms * kMergeGridPerSm));
     int batch = max_chunks <= 4 ? 4 : max_chunks <= 8 ? 8 : max_chunks <= 16 ? 16 : 32;
     int64_t grid = want;
+    // Rows of more than 32 items need the 32-item variant (two (m, l) per lane).
+    const int min_batch = max_chunks > 32 ? 32 : 4;
     for (;; batch /= 2) {
         const int regs = D == 128 ? merge_registers<128>(batch) : merge_registers<64>(batch);
         const int64_t per_sub = (kRegistersPerSubpartition - split_regs_per_subpartition) /
                                 (warp_register_allocation(regs) * kMergeWarps);
         const int64_t fit = (int64_t)num_sms * std::min<int64_t>(kMergeGridPerSm, 4 * per_sub);
-        if (fit >= want || batch == 4) {
+        if (fit >= want || batch == min_batch) {
             grid = std::max<int64_t>(1, std::min(want, fit));
             break;
         }

@@ -273,7 +273,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     if (cudaError_t e = launch_decode(head_dim, G > 1, false, false, grid, maps[0], maps[1], p, st); e != cudaSuccess)
         return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     if (split_rows)
-        if (cudaError_t e = launch_merge(head_dim, false, kMaxChunks, num_sms, 0, p, st); e != cudaSuccess)
+        if (cudaError_t e = launch_merge(head_dim, false, kChunkCap, num_sms, 0, p, st); e != cudaSuccess)
             return fail(KVC_ERR_CUDA, cudaGetErrorString(e));
     return KVC_OK;
 }

@@ -91,19 +91,21 @@ SMALL = [
     ("gqa7_64", 14, 2, 64, [3, 16, 33, 250]),
     ("gqa8_64", 8, 1, 64, [5, 64, 129]),
     ("gqa2_128", 4, 2, 128, [17, 100, 1000]),
-    # rows longer than a 32-page id window, and longer than 32 items at small splits
+    # rows longer than a 32-page id window, and longer than the item cap at small splits
     ("mha64_long", 8, 8, 64, [3000, 40]),
     ("gqa7_long", 28, 4, 128, [4000, 5]),
 ]
 
 
-@pytest.mark.parametrize("max_items", [2, 3, 7, 12, 20, 32])
+@pytest.mark.parametrize("max_items", [2, 3, 7, 12, 20, 32, 48, 64])
 @pytest.mark.parametrize("Hq,Hkv,d", [(8, 8, 128), (28, 4, 128), (14, 2, 64)])
 def test_merge_batch_variants(Hq, Hkv, d, max_items):
     """The merge pass is compiled for 4, 8, 16 or 32 items in flight and the
     launch picks the smallest that covers the step's longest row: one-page
     items and a longest row of max_items pages exercise each variant, with
-    shorter rows (one item, several items) beside it."""
+    shorter rows (one item, several items) beside it.  These batches have
+    few rows, so rows may hold up to 64 items: 48 and 64 exercise the second
+    (m, l) per lane and a second batch of loads."""
     lens = [16 * max_items - 1, 40, 5, 16 * max(1, max_items // 2)]
     cfg = wl.custom(f"merge{max_items}", 1, Hq, Hkv, d, len(lens), lens=lens, seed=400 + max_items,
                     page_order="shuffled")
