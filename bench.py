@@ -230,15 +230,20 @@ def run_gpu(args, rank, world):
         per_layer = B * (Hq + 2 * Hkv) * d
         d_in = torch.empty(L * per_layer, dtype=torch.bfloat16, device="cuda")
         d_out = torch.empty((L, B, Hq, d), dtype=torch.bfloat16, device="cuda")
-        qs, ks, vs = [], [], []
+
+        def views(d_in, d_out):
+            qs, ks, vs = [], [], []
+            for l in range(L):
+                x = d_in[l * per_layer:(l + 1) * per_layer]
+                qs.append(x[:B * Hq * d].view(B, Hq, d))
+                ks.append(x[B * Hq * d:B * (Hq + Hkv) * d].view(B, Hkv, d))
+                vs.append(x[B * (Hq + Hkv) * d:].view(B, Hkv, d))
+            return qs, ks, vs, [d_out[l] for l in range(L)]
+
+        qs, ks, vs, outs = views(d_in, d_out)
         for l in range(L):
-            x = d_in[l * per_layer:(l + 1) * per_layer]
-            qs.append(x[:B * Hq * d].view(B, Hq, d))
-            ks.append(x[B * Hq * d:B * (Hq + Hkv) * d].view(B, Hkv, d))
-            vs.append(x[B * (Hq + Hkv) * d:].view(B, Hkv, d))
             q, k, v = wl.step_inputs(cfg, 0, l, "cuda")
             qs[l].copy_(q), ks[l].copy_(k), vs[l].copy_(v)
-        outs = [d_out[l] for l in range(L)]
     stream.synchronize()
     log(f"[rank {rank}] setup {time.perf_counter() - t_setup:.1f} s; pool "
         f"{sess.query().pool_bytes / 2**30:.1f} GiB")
@@ -251,13 +256,13 @@ def run_gpu(args, rank, world):
         ids_dev = torch.tensor(sess.seq_ids, dtype=torch.int32, device="cuda")
         kd.kv_cache_device_steps(sess.h, B, True, stream)
 
-        def layers():
+        def layers(v):
             for l in range(L):
-                sess.append_attend(l, qs[l], ks[l], vs[l], outs[l])
+                sess.append_attend(l, v[0][l], v[1][l], v[2][l], v[3][l])
 
         with torch.cuda.stream(stream):
             kd.kv_begin_step_device(sess.h, B, ids_dev, stream)   # eager step: nothing lazy in the capture
-            layers()
+            layers((qs, ks, vs, outs))
         sess.lens += 1
         stream.synchronize()
         n0 = sess.query().kernel_launches
@@ -265,8 +270,15 @@ def run_gpu(args, rank, world):
         with torch.cuda.graph(g_begin, stream=stream):
             kd.kv_begin_step_device(sess.h, B, ids_dev, stream)
         with torch.cuda.graph(g_layers, stream=stream):
-            layers()
+            layers((qs, ks, vs, outs))
         graphs = (g_begin, g_layers, sess.query().kernel_launches - n0)
+        # a second input/output set, so the end-to-end leg can move one step's
+        # inputs and outputs while another step runs
+        d_in2, d_out2 = d_in.clone(), torch.empty_like(d_out)
+        g_layers2 = torch.cuda.CUDAGraph()
+        if not args.no_e2e:
+            with torch.cuda.graph(g_layers2, stream=stream):
+                layers(views(d_in2, d_out2))
 
     def step(events=None):
         """One decode step.  events: per-step event list to time the attention
@@ -346,9 +358,10 @@ def run_gpu(args, rank, world):
 
     # ---- end to end: host inputs -> device -> host outputs, every step: a
     # step's q, k_new, v_new of all layers go over from pinned host memory in
-    # one copy, the step runs as timed above (graph replay, or the host calls
-    # with --host-steps / --unfused) and all layers' outputs come back in one
-    # copy.
+    # one copy and all layers' outputs come back in one copy.  With replayed
+    # graphs the copies run on a second stream, double-buffered: step s+1's
+    # inputs move while step s runs, and step s's outputs once it is done.
+    # With --host-steps / --unfused, or under 1 MB a step, they are serial.
     e2e = None
     if not args.no_e2e:
         h_in = d_in.cpu().pin_memory()
@@ -363,16 +376,55 @@ def run_gpu(args, rank, world):
         if world > 1:
             torch.distributed.barrier()
         w0 = time.perf_counter()
-        with torch.cuda.stream(stream):
+        # (a step that moves under 1 MB is launch-bound: the extra stream
+        # operations of double buffering would cost more than they hide)
+        if graphs is not None and h2d + d2h >= 2**20:
+            copy = torch.cuda.Stream()
+            sets = [(d_in, d_out, graphs[1]), (d_in2, d_out2, g_layers2)]
+            ev_in = [torch.cuda.Event() for _ in range(2)]
+            ev_done = [torch.cuda.Event() for _ in range(2)]
+            ev_out = [torch.cuda.Event() for _ in range(2)]
             s0.record(stream)
+            copy.wait_event(s0)
+            with torch.cuda.stream(copy):
+                d_in.copy_(h_in, non_blocking=True)
+                ev_in[0].record(copy)
             for s in range(args.steps):
+                i = s % 2
                 att = [int(n) + 1 for n in sess.lens]
                 a, p = layer_bytes(cfg, att)
                 e_bytes += L * (a + p)
-                d_in.copy_(h_in, non_blocking=True)
-                step()
-                h_out.copy_(d_out, non_blocking=True)
+                with torch.cuda.stream(stream):
+                    stream.wait_event(ev_in[i])
+                    if s >= 2:
+                        stream.wait_event(ev_out[i])   # step s-2's outputs have left this set
+                    graphs[0].replay()
+                    sets[i][2].replay()
+                    ev_done[i].record(stream)
+                sess.lens += 1
+                with torch.cuda.stream(copy):
+                    if s + 1 < args.steps:
+                        j = 1 - i
+                        if s >= 1:
+                            copy.wait_event(ev_done[j])   # step s-1 has read this set's inputs
+                        sets[j][0].copy_(h_in, non_blocking=True)
+                        ev_in[j].record(copy)
+                    copy.wait_event(ev_done[i])
+                    h_out.copy_(sets[i][1], non_blocking=True)
+                    ev_out[i].record(copy)
+            stream.wait_stream(copy)
             s1.record(stream)
+        else:
+            with torch.cuda.stream(stream):
+                s0.record(stream)
+                for s in range(args.steps):
+                    att = [int(n) + 1 for n in sess.lens]
+                    a, p = layer_bytes(cfg, att)
+                    e_bytes += L * (a + p)
+                    d_in.copy_(h_in, non_blocking=True)
+                    step()
+                    h_out.copy_(d_out, non_blocking=True)
+                s1.record(stream)
         stream.synchronize()
         wall = time.perf_counter() - w0
         e_ms = s0.elapsed_time(s1)
