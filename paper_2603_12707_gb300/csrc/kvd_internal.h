@@ -12,6 +12,7 @@ constexpr int kPageSize = 16;          // tokens per page (the only supported P)
 constexpr int kMaxGroup = 8;           // query heads per KV head handled by one MMA N-tile
 constexpr int kMaxChunks = 64;         // work items per (row, KV head) at most
 constexpr int kChunkCap = 32;          // the usual cap; 64 only when few rows must fill the GPU
+constexpr int kChunkCapGqa = 16;       // GQA: the merge variant for 16 items fits beside the split pass
 constexpr int kMaxItemPages = 1024;    // largest target item size a caller may request
 constexpr int kPatchMax = 1024;        // step entries carried in one launch's parameters
 constexpr int kScatterMax = 2048;      // int32 updates carried in one launch's parameters
