@@ -1,6 +1,7 @@
 // Page-table maintenance, the per-step update and split plan, token writes /
 // reads into pages, and the fused K+V append (kv_append).
 #include <algorithm>
+#include <climits>
 
 #include "kvd_internal.h"
 #include "kvd_ptx.cuh"
@@ -46,10 +47,44 @@ __device__ int block_exclusive_scan(int v, int* total)
     return before_warp + x - v;
 }
 
+// Split plan of a step, built by one block of 1024 threads: plan position i
+// takes batch row b, sequence seq, len tokens from row_at(i, &b, &seq, &len);
+// the row is cut into row_chunks() items of near-equal size, a row's items
+// adjacent, its target size graduated by position (row_item_pages).  Entries
+// past max_entries are dropped with error bit 4.  Returns the entries planned.
+template <class RowAt>
+__device__ int build_split_plan(int batch, int item_pages, int chunk_cap, int max_entries, RowAt row_at,
+                                PlanEntry* plan, int2* rows, int32_t* err)
+{
+    int carry = 0;
+    for (int base = 0; base < batch; base += blockDim.x) {
+        const int i = base + threadIdx.x;
+        int b = 0, seq = 0, len = 0, np = 0, nch = 0;
+        if (i < batch) {
+            row_at(i, &b, &seq, &len);
+            np = (len + kPageSize - 1) / kPageSize;
+            nch = row_chunks(np, row_item_pages(item_pages, i, batch), chunk_cap);
+        }
+        int total;
+        const int off = carry + block_exclusive_scan(nch, &total);
+        if (off + nch > max_entries) {
+            flag_error(err, 4);
+            nch = 0;
+        }
+        for (int c = 0; c < nch; ++c) {
+            int first, n;
+            chunk_range(np, nch, c, &first, &n);
+            plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
+        }
+        if (i < batch) rows[b] = make_int2(off, nch);
+        carry += total;
+    }
+    return carry;
+}
+
 // Apply the step's length / page-table updates; in the last launch of a step,
-// build the split plan: rows in the host's order (longest first when the
-// batch fits one launch), each row cut into row_chunks() items of near-equal
-// size, a row's items adjacent.
+// build the split plan with the rows in the host's order (longest first when
+// the batch fits one launch).  The host sized the plan for exactly this step.
 __global__ void __launch_bounds__(1024)
     step_kernel(const __grid_constant__ StepPatch patch, const __grid_constant__ PlanArgs a)
 {
@@ -62,31 +97,18 @@ __global__ void __launch_bounds__(1024)
     }
     if (!a.build) return;
     __syncthreads();
-    int carry = 0;
-    for (int base = 0; base < a.batch; base += blockDim.x) {
-        const int i = base + threadIdx.x;
-        int b = 0, seq = 0, len = 0, np = 0, nch = 0;
-        if (i < a.batch) {
-            b = a.use_order ? a.order[i] : i;
-            seq = a.step_seq[b];
-            len = a.seq_len[seq];
-            if (len <= 0 || len > a.max_pages * kPageSize) {
+    build_split_plan(
+        a.batch, a.item_pages, a.chunk_cap, INT_MAX,
+        [&](int i, int* b, int* seq, int* len) {
+            *b = a.use_order ? a.order[i] : i;
+            *seq = a.step_seq[*b];
+            *len = a.seq_len[*seq];
+            if (*len <= 0 || *len > a.max_pages * kPageSize) {
                 flag_error(a.err, 4);
-                len = 1;
+                *len = 1;
             }
-            np = (len + kPageSize - 1) / kPageSize;
-            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch), a.chunk_cap);
-        }
-        int total;
-        const int off = carry + block_exclusive_scan(nch, &total);
-        for (int c = 0; c < nch; ++c) {
-            int first, n;
-            chunk_range(np, nch, c, &first, &n);
-            a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
-        }
-        if (i < a.batch) a.rows[b] = make_int2(off, nch);
-        carry += total;
-    }
+        },
+        a.plan, a.rows, a.err);
 }
 
 // The same step on the device (graph-replayable, no host input): rows in
@@ -159,32 +181,15 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
         }
         __syncthreads();
     }
-    carry = 0;
-    for (int base = 0; base < a.batch; base += blockDim.x) {
-        const int i = base + threadIdx.x;
-        const int b = (ordered && i < a.batch) ? s_order[i] : i;
-        int seq = 0, len = 0, np = 0, nch = 0;
-        if (i < a.batch) {
-            seq = a.step_seq[b];
-            len = max(1, a.seq_len[seq]);
-            np = (len + kPageSize - 1) / kPageSize;
-            nch = row_chunks(np, row_item_pages(a.item_pages, i, a.batch), a.chunk_cap);
-        }
-        int total;
-        const int off = carry + block_exclusive_scan(nch, &total);
-        if (off + nch > a.max_entries) {
-            flag_error(a.err, 4);
-            nch = 0;
-        }
-        for (int c = 0; c < nch; ++c) {
-            int first, n;
-            chunk_range(np, nch, c, &first, &n);
-            a.plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
-        }
-        if (i < a.batch) a.rows[b] = make_int2(off, nch);
-        carry += total;
-    }
-    if (threadIdx.x == 0) *a.n_entries = min(carry, a.max_entries);
+    const int entries = build_split_plan(
+        a.batch, a.item_pages, a.chunk_cap, a.max_entries,
+        [&](int i, int* b, int* seq, int* len) {
+            *b = ordered ? s_order[i] : i;
+            *seq = a.step_seq[*b];
+            *len = max(1, a.seq_len[*seq]);   // 0 only after a failed allocation (error bit 8)
+        },
+        a.plan, a.rows, a.err);
+    if (threadIdx.x == 0) *a.n_entries = min(entries, a.max_entries);
 }
 
 // One thread per 16-byte chunk of a [n][H_kv][D] token block.

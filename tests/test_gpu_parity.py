@@ -91,6 +91,11 @@ SMALL = [
     ("gqa7_64", 14, 2, 64, [3, 16, 33, 250]),
     ("gqa8_64", 8, 1, 64, [5, 64, 129]),
     ("gqa2_128", 4, 2, 128, [17, 100, 1000]),
+    # the other group sizes the MMA tile pads to 8 query heads
+    ("gqa3_64", 6, 2, 64, [2, 31, 160]),
+    ("gqa4_128", 16, 4, 128, [16, 65, 333]),
+    ("gqa5_128", 10, 2, 128, [1, 48, 511]),
+    ("gqa6_64", 12, 2, 64, [9, 80, 257]),
     # rows longer than a 32-page id window, and longer than the item cap at small splits
     ("mha64_long", 8, 8, 64, [3000, 40]),
     ("gqa7_long", 28, 4, 128, [4000, 5]),
