@@ -69,7 +69,20 @@ def layer_bytes(cfg, attended):
 def describe(cfg):
     return {"workload": cfg.name + ": " + cfg.description, "batch": cfg.batch, "layers": cfg.num_layers,
             "layer_pools": cfg.phys_layers, "q_heads": cfg.num_q_heads, "kv_heads": cfg.num_kv_heads,
-            "head_dim": cfg.head_dim, "page_size": cfg.page_size, "seed": cfg.seed}
+            "head_dim": cfg.head_dim, "page_size": cfg.page_size, "page_order": cfg.page_order,
+            "seed": cfg.seed}
+
+
+def workload_config(args):
+    """The named workload with the command line's overrides (layer pools held, page order)."""
+    import dataclasses
+    from paper_2603_12707_gb300 import workloads as wl
+    cfg = wl.CONFIGS[args.config]
+    if args.phys_layers:
+        cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
+    if args.page_order:
+        cfg = dataclasses.replace(cfg, page_order=args.page_order)
+    return cfg
 
 
 # ------------------------------------------------------------------ clocks
@@ -211,10 +224,7 @@ def run_gpu(args, rank, world):
         _build.build_library()
     if world > 1:
         torch.distributed.barrier()
-    cfg = wl.CONFIGS[args.config]
-    if args.phys_layers:
-        import dataclasses
-        cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
+    cfg = workload_config(args)
     stream = torch.cuda.Stream()
     total_steps = args.warmup + args.steps + (args.steps if not args.no_e2e else 0) + 2
     t_setup = time.perf_counter()
@@ -452,10 +462,7 @@ def run_varlen_write(args, rank, world):
         _build.build_library()
     if world > 1:
         torch.distributed.barrier()
-    cfg = wl.CONFIGS[args.config]
-    if args.phys_layers:
-        import dataclasses
-        cfg = dataclasses.replace(cfg, phys_layers=args.phys_layers)
+    cfg = workload_config(args)
     stream = torch.cuda.Stream()
     sess = DecodeSession(cfg, extra_tokens=1, device="cuda", stream=stream)
     lens = [int(n) for n in sess.lens0]
@@ -545,6 +552,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="llava", choices=["tiny", "llava", "qwen", "ragged", "long"])
     ap.add_argument("--phys-layers", type=int, default=0, help="layer pools held (profiling on a smaller cache)")
+    ap.add_argument("--page-order", choices=["sequential", "shuffled", "interleaved"], default=None,
+                    help="physical page order of the pool (default: the workload's own)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--split-pages", type=int, default=0,
                     help="target pages per work item (0: the library's automatic choice)")
@@ -615,7 +624,10 @@ def main():
     attn_bytes = statistics.mean(r["attn_bytes"])
     peak, peak_kind = measured_peaks()
     achieved = attn_bytes / (attn_ms / 1e3) / 1e9
-    traffic = None if args.unfused else committed_traffic(KERNEL_SOURCES, cfg.name, attn_bytes)
+    # the committed captures were taken with each workload's own page order
+    default_order = args.page_order in (None, wl.CONFIGS[args.config].page_order)
+    traffic = (committed_traffic(KERNEL_SOURCES, cfg.name, attn_bytes)
+               if not args.unfused and default_order else None)
     out = {
         "metric": METRIC, "value": round(gbs, 2), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
