@@ -8,8 +8,9 @@
 //     covering K and V (128-byte swizzle, L2 evict-first), completing on one
 //     mbarrier per stage;
 //   * the warp computes an online softmax over the item's tokens for the G
-//     query heads of the KV head (running max m in log2 units, running sum l,
-//     unnormalised accumulator o, all fp32);
+//     query heads of the KV head (reference max m in log2 units, running sum
+//     l = sum 2^(s - m), unnormalised accumulator o, all fp32; MHA keeps m at
+//     the running max, GQA lets it trail the running max by up to 8);
 //   * a row with one item writes bf16 output directly; otherwise each item
 //     stores (o, m, l) as a partial and a second pass (merge_kernel in
 //     kvd_merge.cu, one warp
@@ -226,15 +227,27 @@ struct GqaCompute {
     __device__ __forceinline__ void page(uint8_t*, uint8_t* sVp, uint32_t sK, uint32_t sV, int valid,
                                          float scale_log2, int lane)
     {
+        // S^T over the D/16 k-steps in four independent accumulator chains
+        // (a shorter dependent MMA sequence), summed at the end.
         float sc[4] = {0.f, 0.f, 0.f, 0.f};
         {
+            constexpr int NA = KS < 4 ? KS : 4;
+            float acc[NA][4];
+#pragma unroll
+            for (int a = 0; a < NA; ++a)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) acc[a][k] = 0.f;
             const int r = (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
             for (int ks = 0; ks < KS; ++ks) {
                 uint32_t a0, a1, a2, a3;
                 ldsm_x4(sK + swz(r, ks * 2 + (lane >> 4)), a0, a1, a2, a3);
-                mma_bf16_16816(sc, a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
+                mma_bf16_16816(acc[ks % NA], a0, a1, a2, a3, qb[ks][0], qb[ks][1]);
             }
+#pragma unroll
+            for (int a = 0; a < NA; ++a)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) sc[k] += acc[a][k];
         }
         const int t0 = lane >> 2, t1 = t0 + 8;
         const bool v0 = t0 < valid, v1 = t1 < valid;
@@ -242,27 +255,37 @@ struct GqaCompute {
         sc[1] = v0 ? sc[1] * scale_log2 : -INFINITY;
         sc[2] = v1 ? sc[2] * scale_log2 : -INFINITY;
         sc[3] = v1 ? sc[3] * scale_log2 : -INFINITY;
+        // The reference m of a head moves only when one of its scores exceeds
+        // it by more than 8 (log2 units): the weights 2^(s - m) then stay at
+        // most 2^8, far inside the fp32 and bf16 range, and most pages skip
+        // the max reduction and the rescale of o and l.  Any reference gives
+        // the same o / l; the merge pass takes (o, m, l) with m as that
+        // reference.
         float pm0 = fmaxf(sc[0], sc[2]), pm1 = fmaxf(sc[1], sc[3]);
+        if (__any_sync(0xffffffffu, pm0 > m0 + 8.f || pm1 > m1 + 8.f)) {
 #pragma unroll
-        for (int mask = 4; mask < 32; mask <<= 1) {
-            pm0 = fmaxf(pm0, __shfl_xor_sync(0xffffffffu, pm0, mask));
-            pm1 = fmaxf(pm1, __shfl_xor_sync(0xffffffffu, pm1, mask));
-        }
-        const float mn0 = fmaxf(m0, pm0), mn1 = fmaxf(m1, pm1);
-        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
-        const float p0 = ex2(sc[0] - mn0), p1 = ex2(sc[1] - mn1);
-        const float p2 = ex2(sc[2] - mn0), p3 = ex2(sc[3] - mn1);
-        l0 = fmaf(l0, al0, p0 + p2);
-        l1 = fmaf(l1, al1, p1 + p3);
-        m0 = mn0;
-        m1 = mn1;
+            for (int mask = 4; mask < 32; mask <<= 1) {
+                pm0 = fmaxf(pm0, __shfl_xor_sync(0xffffffffu, pm0, mask));
+                pm1 = fmaxf(pm1, __shfl_xor_sync(0xffffffffu, pm1, mask));
+            }
+            const float mn0 = fmaxf(m0, pm0), mn1 = fmaxf(m1, pm1);
+            const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+            l0 *= al0;
+            l1 *= al1;
+            m0 = mn0;
+            m1 = mn1;
 #pragma unroll
-        for (int mt = 0; mt < KS; ++mt) {
-            oacc[mt][0] *= al0;
-            oacc[mt][1] *= al1;
-            oacc[mt][2] *= al0;
-            oacc[mt][3] *= al1;
+            for (int mt = 0; mt < KS; ++mt) {
+                oacc[mt][0] *= al0;
+                oacc[mt][1] *= al1;
+                oacc[mt][2] *= al0;
+                oacc[mt][3] *= al1;
+            }
         }
+        const float p0 = ex2(sc[0] - m0), p1 = ex2(sc[1] - m1);
+        const float p2 = ex2(sc[2] - m0), p3 = ex2(sc[3] - m1);
+        l0 += p0 + p2;
+        l1 += p1 + p3;
         // P^T as the B operand: lane needs P[t=2(lane&3)+{0,1}][h=lane>>2] and
         // the same for t+8.  P[t][h] for t < 8 sits in lane 4t + h/2.
         const int srcA = 8 * (lane & 3) + (lane >> 3);
