@@ -212,8 +212,9 @@ KVC_API int kv_append(kv_cache *cache, int32_t layer, int32_t batch, const void 
  * same layer first, on the same stream.  softmax_scale <= 0 selects
  * 1/sqrt(d_h).  Split-KV: the step's plan cuts each (sequence, KV head) into
  * work items of consecutive pages; each item runs an online softmax in fp32
- * over its pages for all G query heads of the KV head, and the last item of a
- * (sequence, KV head) to finish merges the partial results by log-sum-exp. */
+ * over its pages for all G query heads of the KV head, and a second kernel
+ * merges the partial results of every (sequence, KV head) cut into several
+ * items by log-sum-exp. */
 KVC_API int decode_attention(kv_cache *cache, int32_t layer, int32_t batch, const void *q, void *out,
                      float softmax_scale, void *stream);
 
