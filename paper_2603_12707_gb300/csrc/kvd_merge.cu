@@ -75,12 +75,14 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
     float M = kTwoSlots ? fmaxf(ml0.x, ml1.x) : ml0.x;
 #pragma unroll
     for (int o = 16; o; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    // Items lane and lane + 32 weigh e = 2^(m - M); the sum of e * o is
+    // divided by L = sum e * l at the end, so the reduction of L runs beside
+    // the weighted sum instead of before it.
     const float e0 = (lane < nch) ? ex2(ml0.x - M) : 0.f;
     const float e1 = (kTwoSlots && lane + 32 < nch) ? ex2(ml1.x - M) : 0.f;
     float L = kTwoSlots ? e0 * ml0.y + e1 * ml1.y : e0 * ml0.y;
 #pragma unroll
     for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    const float w0 = e0 / L, w1 = e1 / L;   // weights of items lane and lane + 32
     float acc[PER];
 #pragma unroll
     for (int j = 0; j < PER; ++j) acc[j] = 0.f;
@@ -88,11 +90,14 @@ __device__ __forceinline__ void merge_unit(const DecodeParams& p, int2 row, int 
         if (c0) load(c0);
 #pragma unroll
         for (int u = 0; u < BATCH; ++u) {
-            const float wc = __shfl_sync(0xffffffffu, (!kTwoSlots || c0 + u < 32) ? w0 : w1, (c0 + u) & 31);
+            const float wc = __shfl_sync(0xffffffffu, (!kTwoSlots || c0 + u < 32) ? e0 : e1, (c0 + u) & 31);
 #pragma unroll
             for (int j = 0; j < PER; ++j) acc[j] = fmaf(wc, vals[u][j], acc[j]);
         }
     }
+    const float inv = 1.f / L;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) acc[j] *= inv;
     uint16_t* orow = p.out + ((int64_t)b * p.H_q + g * p.G + hh) * D + d0;
     if constexpr (PER == 4) {
         *reinterpret_cast<uint2*>(orow) = make_uint2(pack_bf16(acc[0], acc[1]), pack_bf16(acc[2], acc[3]));

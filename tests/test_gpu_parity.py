@@ -153,6 +153,23 @@ def test_custom_softmax_scale():
     t.close()
 
 
+@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("split", [0, 1, 3])
+@pytest.mark.parametrize("Hq,Hkv,d", [(28, 4, 128), (8, 8, 64), (6, 2, 64)])
+def test_wide_score_range_moves_the_running_max(Hq, Hkv, d, split, fused):
+    """softmax_scale 3 makes the scores N(0, (3 sqrt(d))^2): the running max of
+    a head keeps jumping by far more than 2^8 across pages and items, so every
+    rescale path of the split pass and the merge runs."""
+    cfg = wl.custom("wide", 1, Hq, Hkv, d, 3, lens=[300, 700, 47], seed=41 + d, page_order="shuffled")
+    t = Tracked(cfg, split_pages=split)
+    t.begin_step()
+    out, q, _, _ = t.run_layer(0, scale=3.0, fused=fused)
+    torch.cuda.synchronize()
+    ref, vmax = t.oracle(0, q, scale=3.0)
+    assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv, what=(Hq, Hkv, d, split, fused))
+    t.close()
+
+
 def test_single_token_context_returns_appended_v():
     """A sequence with nothing cached attends only its new token: out == v_new
     exactly (weights are exactly 1, and bf16 -> fp32 -> bf16 is lossless)."""
