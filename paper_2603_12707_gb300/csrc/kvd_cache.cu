@@ -51,11 +51,16 @@ __device__ int block_exclusive_scan(int v, int* total)
 // takes batch row b, sequence seq, len tokens from row_at(i, &b, &seq, &len);
 // the row is cut into row_chunks() items of near-equal size, a row's items
 // adjacent, its target size graduated by position (row_item_pages).  Entries
-// past max_entries are dropped with error bit 4.  Returns the entries planned.
+// past max_entries are dropped with error bit 4.  Each entry's page ids are
+// copied from the page table into pages_out (stride page_stride), so the
+// decode kernel reads them alongside the entry.  Returns the entries planned.
 template <class RowAt>
 __device__ int build_split_plan(int batch, int item_pages, int chunk_cap, int max_entries, RowAt row_at,
-                                PlanEntry* plan, int2* rows, int32_t* err)
+                                PlanEntry* plan, int2* rows, const int32_t* page_table, int max_pages,
+                                int32_t* pages_out, int page_stride, int32_t* err)
 {
+    __shared__ int s_seq[1024], s_np[1024], s_off[1024], s_nch[1024];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     int carry = 0;
     for (int base = 0; base < batch; base += blockDim.x) {
         const int i = base + threadIdx.x;
@@ -77,6 +82,51 @@ __device__ int build_split_plan(int batch, int item_pages, int chunk_cap, int ma
             plan[off + c] = PlanEntry{b, seq, len, first, n, c, nch, off};
         }
         if (i < batch) rows[b] = make_int2(off, nch);
+        s_seq[threadIdx.x] = seq;
+        s_np[threadIdx.x] = np;
+        s_off[threadIdx.x] = off;
+        s_nch[threadIdx.x] = nch;
+        __syncthreads();
+        // Page ids: each row gets (warps / rows) warps, at least one; a warp
+        // copies 32-page windows of its row, four windows in flight per lane.
+        // Page j of a row lies in item c at offset o (chunk_range inverted:
+        // the first np % nch items hold one page more).
+        const int n_rows = min((int)blockDim.x, batch - base);
+        const int n_warps = (int)(blockDim.x >> 5);
+        const int per_row = n_rows >= n_warps ? 1 : n_warps / n_rows;
+        for (int t = warp; t < n_rows * per_row; t += n_warps) {
+            const int r = t / per_row, part = t - r * per_row;
+            const int rnp = s_np[r], rnch = s_nch[r];
+            if (rnch == 0) continue;
+            const int small = rnp / rnch, extra = rnp % rnch, big_pages = extra * (small + 1);
+            const int32_t* src = page_table + (int64_t)s_seq[r] * max_pages;
+            for (int w0 = part; w0 * 32 < rnp; w0 += 4 * per_row) {
+                int32_t v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int j = (w0 + u * per_row) * 32 + lane;
+                    v[u] = j < rnp ? src[j] : 0;
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int j = (w0 + u * per_row) * 32 + lane;
+                    if (j >= rnp) continue;
+                    int c, o;
+                    if (j < big_pages) {
+                        c = j / (small + 1);
+                        o = j - c * (small + 1);
+                    } else {
+                        c = extra + (j - big_pages) / small;
+                        o = j - big_pages - (c - extra) * small;
+                    }
+                    if (o < page_stride)
+                        pages_out[(int64_t)(s_off[r] + c) * page_stride + o] = v[u];
+                    else
+                        flag_error(err, 4);
+                }
+            }
+        }
+        __syncthreads();   // the next chunk of rows reuses the shared arrays
         carry += total;
     }
     return carry;
@@ -108,7 +158,7 @@ __global__ void __launch_bounds__(1024)
                 *len = 1;
             }
         },
-        a.plan, a.rows, a.err);
+        a.plan, a.rows, a.page_table, a.max_pages, a.page_ids, a.page_stride, a.err);
 }
 
 // The same step on the device (graph-replayable, no host input): rows in
@@ -188,7 +238,7 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
             *seq = a.step_seq[*b];
             *len = max(1, a.seq_len[*seq]);   // 0 only after a failed allocation (error bit 8)
         },
-        a.plan, a.rows, a.err);
+        a.plan, a.rows, a.page_table, a.max_pages, a.page_ids, a.page_stride, a.err);
     if (threadIdx.x == 0) *a.n_entries = min(entries, a.max_entries);
 }
 

@@ -748,6 +748,8 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         pa.plan = c->plan;
         pa.rows = c->rows;
         pa.chunk_cap = cap;
+        pa.page_ids = c->item_pages;
+        pa.page_stride = stride;
         pa.err = c->err;
         // Longest rows first: their items start early and the tail is short.
         pa.use_order = use_order ? 1 : 0;
@@ -766,9 +768,6 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
             KVD_CUDA(launch_step(patch, pa, st));
             ++c->launches;
         }
-        KVD_CUDA(launch_gather_pages(c->plan, (int32_t)entries, nullptr, c->page_table(), c->cfg.max_pages_per_seq,
-                                     c->item_pages, stride, c->num_sms, st));
-        ++c->launches;
     }
     if (!c->host_only)
         if (int rc = push_free_stack(c, static_cast<cudaStream_t>(stream))) return rc;
@@ -947,11 +946,10 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     a.rows = c->rows;
     a.n_entries = c->d_small + 1;
     a.chunk_cap = c->dev_chunk_cap;
+    a.page_ids = c->item_pages;
+    a.page_stride = c->dev_stride;
     a.err = c->err;
     KVD_CUDA(launch_step_device(a, st));
-    ++c->launches;
-    KVD_CUDA(launch_gather_pages(c->plan, c->dev_entries_cap, c->d_small + 1, c->page_table(),
-                                 c->cfg.max_pages_per_seq, c->item_pages, c->dev_stride, c->num_sms, st));
     ++c->launches;
     c->dev_dirty = true;
     c->step_active = true;

@@ -82,6 +82,8 @@ struct PlanArgs {
     PlanEntry* plan;     // [n_entries]
     int2* rows;          // [batch]: (first partial slot, items) of each batch row
     int32_t chunk_cap;   // items per row at most (kChunkCap or kMaxChunks)
+    int32_t* page_ids;   // [entries][page_stride]: page ids of each entry's pages
+    int32_t page_stride;
     int32_t* err;
 };
 
@@ -101,6 +103,8 @@ struct StepDevArgs {
     int2* rows;
     int32_t* n_entries;       // out: plan entries of the step
     int32_t chunk_cap;        // items per row at most (kChunkCap or kMaxChunks)
+    int32_t* page_ids;        // [max_entries][page_stride]: page ids of each entry's pages
+    int32_t page_stride;
     int32_t* err;
 };
 
