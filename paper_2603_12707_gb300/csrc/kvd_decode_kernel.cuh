@@ -13,9 +13,8 @@
 //     the running max, GQA lets it trail the running max by up to 8);
 //   * a row with one item writes bf16 output directly; otherwise each item
 //     stores (o, m, l) as a partial and a second pass (merge_kernel in
-//     kvd_merge.cu, one warp
-//     per (row, query head), one lane per item's (m, l), every item's o in
-//     flight at once) merges them by log-sum-exp:
+//     kvd_merge.cu: one warp per (row, query head), one lane per item's
+//     (m, l), every item's o in flight at once) merges them by log-sum-exp:
 //         M = max_c m_c,  O = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c.
 // MHA (G = 1, 1 flop per byte) runs on the CUDA cores; GQA (2 <= G <= 8) runs
 // Q.K^T and P.V as m16n8k16 bf16 MMAs with the 16 tokens of a page as M and the
@@ -39,7 +38,6 @@ namespace kvd {
 
 namespace {
 
-
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
@@ -47,8 +45,8 @@ template <int D, bool GQA>
 struct Geo {
     static constexpr int kTileBytes = kPageSize * D * 2; // one (page, head) tile
     static constexpr int kStageBytes = 2 * kTileBytes;   // K tile + V tile
-    // stages per warp (8 one-warp CTAs per SM); deeper rings with fewer warps
-    // measured slower for both paths
+    // stages per warp (8 one-warp CTAs per SM at d = 128); deeper rings with
+    // fewer warps, and for GQA a 2-stage ring with 12 warps, measured slower
     static constexpr int kRing = D == 128 ? 3 : 6;
     static constexpr int kRingBytes = kWarps * kRing * kStageBytes;
     static constexpr int kSmem = kRingBytes + kWarps * kRing * 8 + 1024;
