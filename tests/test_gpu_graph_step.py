@@ -204,3 +204,30 @@ def test_host_step_cannot_move_buffers_under_device_steps(kvlib):
     kd.kv_begin_step(h, seqs)
     assert [kd.kv_seq_info(h, s_)[0] for s_ in seqs] == [1901] * 4
     kd.kv_cache_destroy(h)
+
+
+def test_batch_beyond_one_block_device_and_host_steps(kvlib):
+    """1100 rows: the step kernels plan and copy page lists in two chunks of
+    1024 rows (the host step also takes two launches); device and host steps
+    give bit-identical outputs, and rows from both chunks match the oracle."""
+    rng = np.random.default_rng(11)
+    lens = [int(x) for x in rng.integers(0, 90, 1100)]
+    cfg = wl.custom("wide_batch", 1, 8, 2, 64, 1100, lens=lens, seed=19, page_order="shuffled")
+    keep = [0, 1, 500, 1023, 1024, 1025, 1099]
+    a = Tracked(cfg, extra_tokens=6, split_pages=SPLIT, keep_host=True, keep_rows=keep)
+    b = Tracked(cfg, extra_tokens=6, split_pages=SPLIT, keep_host=False)
+    kd.kv_cache_device_steps(b.sess.h, cfg.batch)
+    ids = torch.tensor(b.sess.seq_ids, dtype=torch.int32, device="cuda")
+    for step in range(3):
+        a.begin_step()
+        kd.kv_begin_step_device(b.sess.h, cfg.batch, ids)
+        b.step += 1
+        b.sess.lens += 1
+        oa, q, _, _ = a.run_layer(0, fused=True)
+        ob, _, _, _ = b.run_layer(0, fused=True)
+        torch.cuda.synchronize()
+        assert torch.equal(oa, ob), step
+        ref, vmax = a.oracle(0, q, rows=keep)
+        assert_close(bf16_to_f64(ob)[keep], ref, vmax, gqa=True, what=step)
+    a.close()
+    b.close()
