@@ -261,7 +261,10 @@ KVC_API int kv_cache_device_steps(kv_cache *cache, int32_t max_batch, int32_t en
  * ([batch] distinct live sequence ids, read when the kernel runs, so a
  * replayed graph may change them between replays); pages come off the
  * device free stack in batch order, exactly as kv_begin_step takes them.
- * A pool that runs out sets KVC_DEVERR_OOM (the row keeps its length).  No
+ * A pool that runs out sets KVC_DEVERR_OOM, a sequence id outside the cache
+ * or a full page row KVC_DEVERR_SEQ_RANGE; such a row keeps its length, and
+ * the layer calls of the step (kv_append, decode_attention,
+ * decode_attention_append) leave its cache and its output row untouched.  No
  * host synchronisation; graph-capturable. */
 KVC_API int kv_begin_step_device(kv_cache *cache, int32_t batch, const int32_t *seq_ids, void *stream);
 

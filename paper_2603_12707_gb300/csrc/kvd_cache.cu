@@ -166,26 +166,35 @@ __global__ void __launch_bounds__(1024)
 // the next page of the device free stack, in batch order (the same pages the
 // host allocator would hand out); then the split plan, rows longest first
 // (stable, as on the host) when the batch fits one block, else in batch order.
+// A row whose step fails (a sequence id outside [0, max_seqs), a full page
+// row, or an exhausted pool: error bits 4 / 8) keeps its length and gets
+// step_seq -1 and no work items, so the layer calls that follow neither write
+// its cache nor its output row.  With the batch in one block, each row's
+// sequence and new length stay in shared memory for the ranking and the plan.
 __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
 {
     __shared__ int s_top;
+    __shared__ int s_seq[1024], s_len[1024];   // per batch row when the batch fits the block
+    const bool small = a.batch <= (int)blockDim.x;
     if (threadIdx.x == 0) s_top = *a.free_top;
-    __syncthreads();
-    const int top0 = s_top;
+    int top0 = 0;
     int carry = 0;
     for (int base = 0; base < a.batch; base += blockDim.x) {
         const int i = base + threadIdx.x;
-        int seq = 0, len = 0, need = 0;
+        int seq = -1, len = 0, need = 0;
         bool ok = false;
         if (i < a.batch) {
             seq = a.seq_ids[i];
-            len = a.seq_len[seq];
-            ok = len >= 0 && len + 1 <= a.max_pages * kPageSize;
+            if (seq >= 0 && seq < a.max_seqs) {
+                len = a.seq_len[seq];
+                ok = len >= 0 && len + 1 <= a.max_pages * kPageSize;
+            }
             if (!ok) flag_error(a.err, 4);
             need = (ok && len % kPageSize == 0) ? 1 : 0;
         }
         int total;
-        const int rank = carry + block_exclusive_scan(need, &total);
+        const int rank = carry + block_exclusive_scan(need, &total);   // also orders s_top's write
+        if (base == 0) top0 = s_top;
         if (ok) {
             int32_t page = -1;
             if (need) {
@@ -200,24 +209,30 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
             if (ok) {
                 if (page >= 0) a.page_table[(int64_t)seq * a.max_pages + len / kPageSize] = page;
                 a.seq_len[seq] = len + 1;
+                len += 1;
             }
         }
-        if (i < a.batch) a.step_seq[i] = seq;
+        if (i < a.batch) {
+            a.step_seq[i] = ok ? seq : -1;
+            if (small) {
+                s_seq[i] = ok ? seq : -1;
+                s_len[i] = ok ? len : 0;
+            }
+        }
         carry += total;
     }
     __syncthreads();
     if (threadIdx.x == 0) *a.free_top = top0 - min(carry, top0);
 
     // Row order: the rank of row b counts the rows with more pages, and the
-    // rows with as many pages that come before b.
+    // rows with as many pages that come before b (failed rows have none).
     __shared__ int s_np[1024];
     __shared__ int s_order[1024];
-    const bool ordered = a.batch <= (int)blockDim.x;
-    if (ordered) {
+    if (small) {
         const int b = threadIdx.x;
         int np = 0;
         if (b < a.batch) {
-            np = (max(1, a.seq_len[a.step_seq[b]]) + kPageSize - 1) / kPageSize;
+            np = (s_len[b] + kPageSize - 1) / kPageSize;
             s_np[b] = np;
         }
         __syncthreads();
@@ -234,9 +249,10 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
     const int entries = build_split_plan(
         a.batch, a.item_pages, a.chunk_cap, a.max_entries,
         [&](int i, int* b, int* seq, int* len) {
-            *b = ordered ? s_order[i] : i;
-            *seq = a.step_seq[*b];
-            *len = max(1, a.seq_len[*seq]);   // 0 only after a failed allocation (error bit 8)
+            *b = small ? s_order[i] : i;
+            *seq = small ? s_seq[*b] : a.step_seq[*b];
+            *len = *seq < 0 ? 0 : (small ? s_len[*b] : a.seq_len[*seq]);   // 0 tokens: no items
+            if (*seq < 0) *seq = 0;
         },
         a.plan, a.rows, a.page_table, a.max_pages, a.page_ids, a.page_stride, a.err);
     if (threadIdx.x == 0) *a.n_entries = min(entries, a.max_entries);
@@ -349,6 +365,7 @@ __global__ void append_kernel(const AppendArgs a)
     const int g = bg % a.H_kv;
     const int b = bg / a.H_kv;
     const int seq = a.step_seq[b];
+    if (seq < 0) return;   // the row's device-side step failed (already flagged)
     const int pos = a.seq_len[seq] - 1;
     if (pos < 0 || pos >= a.max_pages * kPageSize) {
         flag_error(a.err, 4);

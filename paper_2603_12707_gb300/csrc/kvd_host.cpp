@@ -933,6 +933,7 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     StepDevArgs a;
     a.batch = batch;
+    a.max_seqs = c->cfg.max_seqs;
     a.item_pages = c->dev_item_pages;
     a.max_pages = c->cfg.max_pages_per_seq;
     a.max_entries = c->dev_entries_cap;

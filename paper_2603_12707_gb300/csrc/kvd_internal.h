@@ -90,13 +90,14 @@ struct PlanArgs {
 // kv_begin_step_device: the step's lazy allocation and plan, on the device.
 struct StepDevArgs {
     int32_t batch;
+    int32_t max_seqs;         // sequence ids outside [0, max_seqs) fail their row
     int32_t item_pages;       // target pages per work item (T)
     int32_t max_pages;        // page-table row length
     int32_t max_entries;      // capacity of plan
     const int32_t* seq_ids;   // [batch] sequence ids (device)
     int32_t* free_pages;      // device free stack; the next page is free_pages[*free_top - 1]
     int32_t* free_top;
-    int32_t* step_seq;
+    int32_t* step_seq;        // out: [batch] sequence of each row, -1 where the row's step failed
     int32_t* seq_len;
     int32_t* page_table;
     PlanEntry* plan;

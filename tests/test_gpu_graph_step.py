@@ -108,15 +108,29 @@ def test_captured_step_replays_like_host_steps(kvlib):
 def test_device_step_reports_an_exhausted_pool(kvlib):
     """5 pages, 3 sequences of 16 tokens (3 pages held): the next step needs a
     page for each; the first two rows (batch order) get them, the third is
-    left at its length and the pool exhaustion is reported."""
+    left at its length and the pool exhaustion is reported.  The fused layer
+    launched after it appends the new token of the first two rows and leaves
+    the third row's cache untouched (its last cached token is not
+    overwritten)."""
     cfg = kd.make_config(1, 8, 8, 64, 5, 4, 8)
     h = kd.kv_cache_create(cfg)
     seqs = [kd.kv_seq_create(h) for _ in range(3)]
+    gen = torch.Generator().manual_seed(3)
+    cached = []
     for s_ in seqs:
         kd.kv_seq_reserve(h, s_, 16)
+        k = torch.randn(16, 8, 64, generator=gen).to(torch.bfloat16).cuda()
+        v = torch.randn(16, 8, 64, generator=gen).to(torch.bfloat16).cuda()
+        kd.kv_write_tokens(h, 0, s_, 0, 16, k, v)
+        cached.append((k, v))
     kd.kv_cache_device_steps(h, 3)
     ids = torch.tensor(seqs, dtype=torch.int32, device="cuda")
     kd.kv_begin_step_device(h, 3, ids)
+    q = torch.randn(3, 8, 64, generator=gen).to(torch.bfloat16).cuda()
+    kn = torch.randn(3, 8, 64, generator=gen).to(torch.bfloat16).cuda()
+    vn = torch.randn(3, 8, 64, generator=gen).to(torch.bfloat16).cuda()
+    out = torch.zeros(3, 8, 64, dtype=torch.bfloat16, device="cuda")
+    kd.decode_attention_append(h, 0, 3, q, kn, vn, out)
     torch.cuda.synchronize()
     with pytest.raises(kd.KVDecodeError) as ei:
         kd.kv_cache_query(h)
@@ -135,7 +149,42 @@ def test_device_step_reports_an_exhausted_pool(kvlib):
     m.seq_reserve(1, 1)
     for i, s_ in enumerate(seqs):
         assert kd.kv_seq_info(h, s_)[1] == m.pages[i]
+    for i, s_ in enumerate(seqs):
+        n = 17 if i < 2 else 16
+        k = torch.empty(n, 8, 64, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        kd.kv_read_tokens(h, 0, s_, 0, n, k, v)
+        torch.cuda.synchronize()
+        assert torch.equal(k[:16], cached[i][0]) and torch.equal(v[:16], cached[i][1]), i
+        if i < 2:
+            assert torch.equal(k[16], kn[i]) and torch.equal(v[16], vn[i]), i
     kd.kv_cache_destroy(h)
+
+
+def test_device_step_skips_an_unknown_sequence_id(kvlib):
+    """A device-side sequence id outside the cache sets KVC_DEVERR_SEQ_RANGE;
+    the other rows step and attend as usual (against the oracle)."""
+    cfg = wl.custom("badid", 1, 8, 8, 64, 3, lens=[20, 33, 9], seed=23)
+    t = Tracked(cfg, extra_tokens=4)
+    kd.kv_cache_device_steps(t.sess.h, 3)
+    s0, s1, s2 = t.sess.seq_ids
+    ids = torch.tensor([s0, 77, s2], dtype=torch.int32, device="cuda")
+    kd.kv_begin_step_device(t.sess.h, 3, ids)
+    gen = torch.Generator().manual_seed(4)
+    q3, kn3, vn3 = (torch.randn(3, 8, 64, generator=gen).to(torch.bfloat16).cuda() for _ in range(3))
+    out3 = torch.zeros(3, 8, 64, dtype=torch.bfloat16, device="cuda")
+    kd.decode_attention_append(t.sess.h, 0, 3, q3, kn3, vn3, out3)
+    torch.cuda.synchronize()
+    st = kd.kv_cache_query(t.sess.h, raise_on_device_error=False)
+    assert st.device_error == kd.KVC_DEVERR_SEQ_RANGE
+    assert [kd.kv_seq_info(t.sess.h, s_)[0] for s_ in (s0, s1, s2)] == [21, 33, 10]
+    # launch rows 0 and 2 are sequences 0 and 2, each with its new token
+    for b in (0, 2):
+        for store, val in ((t.k, kn3[b]), (t.v, vn3[b])):
+            store[(0, b)].append(val.view(torch.int16).cpu().numpy().view(np.uint16))
+    ref, vmax = t.oracle(0, q3, rows=[0, 2])
+    assert_close(bf16_to_f64(out3)[[0, 2]], ref, vmax, gqa=False)
+    t.sess.close()
 
 
 def test_device_steps_interleaved_with_host_lifecycle(kvlib):
