@@ -363,8 +363,9 @@ struct GqaCompute {
     }
 };
 
-// The new token of row (en.b, g) into row r of the staged K and V tiles and
-// into the pool (fused append): lanes 0..CH-1 move K, CH..2CH-1 move V.
+// The new token of row (en.b, g) into row r of the staged K and V tiles and,
+// unless its page id is out of range (already recorded), into the pool
+// (fused append): lanes 0..CH-1 move K, CH..2CH-1 move V.
 template <int D>
 __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanEntry& en, int g, int32_t pid,
                                               uint8_t* sK, uint8_t* sV, int lane)
@@ -377,8 +378,10 @@ __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanE
         const int64_t src = ((int64_t)en.b * p.H_kv + g) * D + c * 8;
         const uint4 v = *reinterpret_cast<const uint4*>((is_k ? p.k_new : p.v_new) + src);
         *reinterpret_cast<uint4*>((is_k ? sK : sV) + swz(r, c)) = v;
-        const int64_t dst = (((int64_t)pid * p.H_kv + g) * kPageSize + r) * D + c * 8;
-        *reinterpret_cast<uint4*>((is_k ? p.pool_k : p.pool_v) + dst) = v;
+        if (pid >= 0 && pid < p.num_pages) {
+            const int64_t dst = (((int64_t)pid * p.H_kv + g) * kPageSize + r) * D + c * 8;
+            *reinterpret_cast<uint4*>((is_k ? p.pool_k : p.pool_v) + dst) = v;
+        }
     }
     __syncwarp();
 }
@@ -495,7 +498,7 @@ __global__ void __launch_bounds__(kWarps * 32)
                 // the issue side has not moved past this page's id window
                 if (en.chunk == en.n_chunks - 1 && j == np - 1) {
                     int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
-                    put_new_token<D>(p, en, g, (pid < 0 || pid >= p.num_pages) ? 0 : pid, sK, sK + TILE, lane);
+                    put_new_token<D>(p, en, g, pid, sK, sK + TILE, lane);
                     wrote = true;
                 }
             }
