@@ -1,0 +1,91 @@
+"""Host-side pieces of bench.py, on CPU: the device-code hash that keys the
+committed traffic capture (comment edits keep it, code edits void it), the
+traffic lookup, the clock-log summary, the algorithmic byte count and the
+workload overrides."""
+import argparse
+import json
+import os
+import shutil
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+from paper_2603_12707_gb300 import workloads as wl  # noqa: E402
+
+
+def _copies(tmp_path):
+    out = []
+    for src in bench.KERNEL_SOURCES:
+        dst = tmp_path / os.path.basename(src)
+        shutil.copy(src, dst)
+        out.append(str(dst))
+    return out
+
+
+def test_code_hash_ignores_comments_and_blank_lines(tmp_path):
+    paths = _copies(tmp_path)
+    h0 = bench.kernel_code_hash(paths)
+    assert h0 == bench.kernel_code_hash(bench.KERNEL_SOURCES)
+    with open(paths[0], "a") as f:
+        f.write("\n\n// a new comment line\n   \n")
+    s = open(paths[1]).read()
+    open(paths[1], "w").write(s.replace("#pragma once", "#pragma once   // trailing comment", 1))
+    assert bench.kernel_code_hash(paths) == h0
+
+
+def test_code_hash_changes_with_code(tmp_path):
+    paths = _copies(tmp_path)
+    h0 = bench.kernel_code_hash(paths)
+    s = open(paths[0]).read()
+    assert "kWaitLimitNs = 1000000000ull" in s
+    open(paths[0], "w").write(s.replace("kWaitLimitNs = 1000000000ull", "kWaitLimitNs = 1000000001ull", 1))
+    assert bench.kernel_code_hash(paths) != h0
+
+
+def test_traffic_lookup_needs_the_captured_code(tmp_path, monkeypatch):
+    paths = _copies(tmp_path)
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    rec = {"source_sha256_16": bench.kernel_code_hash(paths),
+           "captures": {"qwen": {"traffic_over_algorithmic": 1.25}}}
+    (prof / "decode_kernel_traffic.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.committed_traffic(paths, "qwen", 1000) == 1250
+    assert bench.committed_traffic(paths, "llava", 1000) is None      # no capture for it
+    s = open(paths[0]).read()
+    open(paths[0], "w").write(s.replace("kWaitLimitNs = 1000000000ull", "kWaitLimitNs = 2000000000ull", 1))
+    assert bench.committed_traffic(paths, "qwen", 1000) is None       # code changed since
+
+
+def test_clock_summary_reads_the_nvidia_smi_log(tmp_path):
+    log = tmp_path / "clocks.csv"
+    log.write_text(
+        "0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active\n"
+        "0, 1980, 2070, 1350.0, 0x4, Not Active, Not Active, Not Active, Active\n"
+        "0, 2070, 2070, 1390.2, 0x4, Not Active, Not Active, Not Active, Active\n"
+        "garbage line\n")
+    c = bench.ClockSampler(0)
+    c.proc, c.path = object(), str(log)
+    s = c.summary()
+    assert s == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    assert not log.exists()
+
+
+def test_layer_bytes_closed_form():
+    cfg = wl.CONFIGS["qwen"]
+    attended = [1, 17, 300]
+    attn, app = bench.layer_bytes(cfg, attended)
+    kv = sum(attended) * 2 * 4 * 128 * 2
+    assert attn == kv + 3 * 28 * 128 * 2 * 2
+    assert app == 3 * 2 * 4 * 128 * 2
+
+
+def test_workload_overrides():
+    a = argparse.Namespace(config="qwen", phys_layers=0, page_order=None)
+    assert bench.workload_config(a) == wl.CONFIGS["qwen"]
+    a = argparse.Namespace(config="qwen", phys_layers=4, page_order="shuffled")
+    cfg = bench.workload_config(a)
+    assert (cfg.phys_layers, cfg.page_order, cfg.num_layers) == (4, "shuffled", 28)
+    assert bench.describe(cfg)["page_order"] == "shuffled"
