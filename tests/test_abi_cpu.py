@@ -203,6 +203,27 @@ def test_begin_step_rejects_duplicates_and_dead_ids_without_changes(kvlib):
     kvlib.kv_cache_destroy(h)
 
 
+def test_begin_step_stops_at_a_full_page_row_without_changes(kvlib):
+    """A row of max_pages pages takes positions up to max_pages * 16 - 1: the
+    step that fills the last slot succeeds, the next one is refused and
+    leaves the lengths and pages of every sequence in the batch as they were."""
+    h = host_cache(kvlib, max_pages=4)
+    a = kvlib.kv_seq_create(h)
+    b = kvlib.kv_seq_create(h)
+    kvlib.kv_seq_reserve(h, a, 63)
+    kvlib.kv_seq_reserve(h, b, 10)
+    kvlib.kv_begin_step(h, [a, b])
+    assert kvlib.kv_seq_info(h, a)[0] == 64 and len(kvlib.kv_seq_info(h, a)[1]) == 4
+    before = [kvlib.kv_seq_info(h, s) for s in (a, b)]
+    free = kvlib.kv_cache_query(h).free_pages
+    with pytest.raises(kvlib.KVDecodeError) as ei:
+        kvlib.kv_begin_step(h, [b, a])
+    assert ei.value.code == kvlib.KVC_ERR_INVALID
+    assert [kvlib.kv_seq_info(h, s) for s in (a, b)] == before
+    assert kvlib.kv_cache_query(h).free_pages == free
+    kvlib.kv_cache_destroy(h)
+
+
 def test_footprint_query_equals_eq1_when_lengths_fill_pages(kvlib):
     # LLaVA-7B shape: the worked example's 704 tokens are 44 whole pages
     cfg = kvlib.make_config(32, 32, 32, 128, 64, 2, 64, flags=kvlib.KVC_FLAG_HOST_ONLY)

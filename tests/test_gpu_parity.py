@@ -142,6 +142,23 @@ def test_decode_matches_oracle_small(name, Hq, Hkv, d, lens, split):
     t.close()
 
 
+@pytest.mark.parametrize("Hq,Hkv,d", [(8, 8, 128), (28, 4, 128), (6, 2, 64)])
+def test_rows_filled_to_the_last_page_slot(Hq, Hkv, d):
+    """Page-table rows of exactly 4 pages: the third step's row 0 attends all
+    64 positions its row can hold (the last slot of the last page)."""
+    cfg = wl.custom("fullrow", 1, Hq, Hkv, d, 3, lens=[61, 13, 47], seed=61 + d)
+    t = Tracked(cfg, extra_tokens=3, split_pages=1)
+    assert t.sess.max_pages == 4
+    for step in range(3):
+        t.begin_step()
+        out, q, _, _ = t.run_layer(0, fused=(step % 2 == 1))
+        torch.cuda.synchronize()
+        ref, vmax = t.oracle(0, q)
+        assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv, what=(step,))
+    assert kd.kv_seq_info(t.sess.h, t.sess.seq_ids[0])[0] == 64
+    t.close()
+
+
 def test_custom_softmax_scale():
     cfg = wl.custom("scale", 1, 14, 2, 128, 3, lens=[10, 40, 90], seed=5)
     t = Tracked(cfg)
