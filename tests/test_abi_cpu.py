@@ -41,6 +41,8 @@ def host_cache(kvlib, num_pages=64, max_seqs=8, max_pages=16, Hq=8, Hkv=8, d=64,
 @pytest.mark.parametrize("field,value,code", [
     ("head_dim", 96, -5), ("page_size", 32, -5), ("num_q_heads", 72, -5),   # G = 9
     ("num_q_heads", 12, -1), ("num_pages", 0, -1), ("max_seqs", 70000, -1), ("flags", 8, -1),
+    # TMA row coordinates (page * H_kv + head) * 16 and page-table indices stay below 2^31
+    ("num_pages", 2**24, -1), ("max_pages_per_seq", 2**28, -1),
 ])
 def test_create_rejects_bad_configs(kvlib, field, value, code):
     cfg = kvlib.make_config(2, 8, 8, 64, 64, 8, 16, flags=kvlib.KVC_FLAG_HOST_ONLY)
