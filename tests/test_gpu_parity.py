@@ -159,14 +159,18 @@ def test_rows_filled_to_the_last_page_slot(Hq, Hkv, d):
     t.close()
 
 
-def test_custom_softmax_scale():
-    cfg = wl.custom("scale", 1, 14, 2, 128, 3, lens=[10, 40, 90], seed=5)
-    t = Tracked(cfg)
+@pytest.mark.parametrize("scale", [0.37, 1e-4])
+@pytest.mark.parametrize("Hq,Hkv", [(14, 2), (8, 8)])
+def test_custom_softmax_scale(Hq, Hkv, scale):
+    """A caller's scale; at 1e-4 every weight is nearly equal and the output is
+    close to the mean of V (the degenerate uniform softmax)."""
+    cfg = wl.custom("scale", 1, Hq, Hkv, 128, 3, lens=[10, 40, 90], seed=5)
+    t = Tracked(cfg, split_pages=2)
     t.begin_step()
-    out, q, _, _ = t.run_layer(0, scale=0.37)
+    out, q, _, _ = t.run_layer(0, scale=scale)
     torch.cuda.synchronize()
-    ref, vmax = t.oracle(0, q, scale=0.37)
-    assert_close(bf16_to_f64(out), ref, vmax, gqa=True)
+    ref, vmax = t.oracle(0, q, scale=scale)
+    assert_close(bf16_to_f64(out), ref, vmax, gqa=Hq > Hkv)
     t.close()
 
 
