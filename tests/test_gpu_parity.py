@@ -96,6 +96,7 @@ SMALL = [
     ("gqa4_128", 16, 4, 128, [16, 65, 333]),
     ("gqa5_128", 10, 2, 128, [1, 48, 511]),
     ("gqa6_64", 12, 2, 64, [9, 80, 257]),
+    ("gqa8_128", 8, 1, 128, [31, 250, 1100]),
     # rows longer than a 32-page id window, and longer than the item cap at small splits
     ("mha64_long", 8, 8, 64, [3000, 40]),
     ("gqa7_long", 28, 4, 128, [4000, 5]),
