@@ -9,8 +9,8 @@
 //     mbarrier per stage;
 //   * the warp computes an online softmax over the item's tokens for the G
 //     query heads of the KV head (reference max m in log2 units, running sum
-//     l = sum 2^(s - m), unnormalised accumulator o, all fp32; MHA keeps m at
-//     the running max, GQA lets it trail the running max by up to 8);
+//     l = sum 2^(s - m), unnormalised accumulator o, all fp32; m trails the
+//     running max by at most 8, so most pages skip the rescale);
 //   * a row with one item writes bf16 output directly; otherwise each item
 //     stores (o, m, l) as a partial and a second pass (merge_kernel in
 //     kvd_merge.cu: one warp per (row, query head), one lane per item's
@@ -134,17 +134,23 @@ struct MhaCompute {
         float sc = part[0] + __shfl_xor_sync(0xffffffffu, part[0], 1);
         const int tok = (c >> 1) * TPI + tsub;
         sc = (tok < valid) ? sc * scale_log2 : -INFINITY;
-        float pm = sc;
+        // The reference m moves only when a score exceeds it by more than 8
+        // (log2 units; see GqaCompute::page), so most pages skip the max
+        // reduction and the rescale.
+        if (__any_sync(0xffffffffu, sc > m + 8.f)) {
+            float pm = sc;
 #pragma unroll
-        for (int mask = 2; mask < 32; mask <<= 1) pm = fmaxf(pm, __shfl_xor_sync(0xffffffffu, pm, mask));
-        const float mn = fmaxf(m, pm);
-        const float alpha = ex2(m - mn);
-        const float pe = ex2(sc - mn);
-        l = fmaf(l, alpha, (c & 1) ? 0.f : pe);
-        m = mn;
-        const uint64_t a2 = f2_pack(alpha, alpha);
+            for (int mask = 2; mask < 32; mask <<= 1) pm = fmaxf(pm, __shfl_xor_sync(0xffffffffu, pm, mask));
+            const float mn = fmaxf(m, pm);
+            const float alpha = ex2(m - mn);
+            l *= alpha;
+            m = mn;
+            const uint64_t a2 = f2_pack(alpha, alpha);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) o2[k] = f2_fma(o2[k], a2, 0ull);
+            for (int k = 0; k < 4; ++k) o2[k] = f2_fma(o2[k], a2, 0ull);
+        }
+        const float pe = ex2(sc - m);
+        l += (c & 1) ? 0.f : pe;
 #pragma unroll
         for (int i = 0; i < IT; ++i) {
             const float pt = __shfl_sync(0xffffffffu, pe, tsub * CH + 2 * i);
