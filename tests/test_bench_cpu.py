@@ -89,3 +89,14 @@ def test_workload_overrides():
     cfg = bench.workload_config(a)
     assert (cfg.phys_layers, cfg.page_order, cfg.num_layers) == (4, "shuffled", 28)
     assert bench.describe(cfg)["page_order"] == "shuffled"
+
+
+def test_clock_records_the_timing_rules_reject():
+    ok = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 5}
+    cap = {"sm_mhz": 1800.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 5}
+    assert not bench.clocks_slowed(ok)
+    assert not bench.clocks_slowed(cap)              # the power cap is kept and noted
+    for r in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
+        assert bench.clocks_slowed({**ok, "reasons": [r]})
+    assert bench.clocks_slowed({**ok, "sm_mhz": 1200.0})   # far below max with no reason: a clock lock
+    assert not bench.clocks_slowed({"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0})
