@@ -202,11 +202,20 @@ KVC_API int kv_begin_step(kv_cache *cache, int32_t batch, const int32_t *seq_ids
 
 /* Fused K+V append for one layer of the current step: writes k_new[b] and
  * v_new[b] (device, [batch][H_kv][d_h] bf16) into position s_b of each
- * sequence of the step.  `batch` must equal the step's batch. */
+ * sequence of the step.  `batch` must equal the step's batch.  Each decode
+ * step adds one token to every request's cache, which holds the K and V of
+ * all its tokens per layer and KV head (Sec. 2 "Language decoding"; what the
+ * cache holds and its size: Sec. 4.1, Eq. 1).  Pools are written in place;
+ * the caller keeps ownership of k_new / v_new, which must be 16-byte aligned.
+ * Errors (no active step, batch mismatch, bad layer or pointer) are reported
+ * before anything is enqueued. */
 KVC_API int kv_append(kv_cache *cache, int32_t layer, int32_t batch, const void *k_new,
               const void *v_new, void *stream);
 
-/* Decode attention for one layer of the current step.  q: device
+/* Decode attention for one layer of the current step: the memory-bound
+ * decode phase that streams each request's KV cache from HBM once per layer
+ * (Sec. 2 "Language decoding"), over a cache laid out as Eq. 1 counts it
+ * (Sec. 4.1), MHA or GQA (Sec. 5.1).  q: device
  * [batch][H_q][d_h] bf16; out: device [batch][H_q][d_h] bf16 (written).
  * Attends over positions 0 .. s_b of each sequence, so call kv_append for the
  * same layer first, on the same stream.  softmax_scale <= 0 selects

@@ -10,7 +10,7 @@ layers, 32 KV heads, d_h = 128, fixed 576 vision tokens) and Qwen2.5-VL-7B
 (Sec. 6.1 "Models"; Sec. 4.2 Table 3 and "Handling dynamic visual token counts").
 The paper's own workload (COCO 2017 val images, one prompt, up to 128 output
 tokens, Sec. 6.1 "Workload") is not available here; these seeded draws stand in
-for it.  Recipe (what the design doc states):
+for it.  Recipe:
 
 * integers (lengths, vision-prefix sizes, page permutations): numpy PCG64
   seeded with ``seed``;

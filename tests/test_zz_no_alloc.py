@@ -30,7 +30,7 @@ def _close(got, ref, vmax, gqa):
     # differ by at most twice that bound
     err = np.abs(got - ref)
     assert err.max() <= 2e-2 and err.mean() <= 2e-3
-    w = (2.0 ** -9 if gqa else 0.0) + 1e-5
+    w = (2.0 ** -8 if gqa else 0.0) + 1e-5
     assert (err <= 2.0 ** -7 * np.abs(ref) + 2 * w * vmax[:, None, None]).all()
 
 
