@@ -301,9 +301,10 @@ KVC_API int kv_cache_sync(kv_cache *cache);
  *                   cleared by this call), or NULL to discard them
  * Work space is a 16 MiB array in this library's device code, held by every
  * GPU that loads the library until the process exits.  batch <= 1024.
- * Work items are enlarged until the split plan and partial results fit the
- * 16 MiB (one item per row needs no partials at all);
- * KVC_ERR_UNSUPPORTED if they still do not fit.  The first call on
+ * Work items are enlarged (doubled, up to 1024 pages each) until the split
+ * plan and partial results fit the 16 MiB (one item per row needs no
+ * partials at all); KVC_ERR_UNSUPPORTED, with nothing enqueued, if they
+ * still do not fit at 1024 pages.  The first call on
  * each device looks up the array's device address (cudaGetSymbolAddress);
  * make that first call before any stream capture.  Every call uses the same
  * array and clears the counters it needs at its start, so calls that overlap

@@ -174,7 +174,8 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     bool split_rows = false;
     int stride = 1;
     size_t off_pages = 0, off_o = 0, off_ml = 0, off_rows = 0, off_q = 0, off_err = 0, need = 0;
-    for (;; T *= 2) {
+    // T doubles, clamped to kMaxItemPages; the attempt at kMaxItemPages is the last.
+    for (;; T = std::min<int64_t>(2 * T, kMaxItemPages)) {
         entries = 0;
         int64_t split_items = 0;   // only rows cut into several items keep partials
         for (int b = 0; b < batch; ++b) {

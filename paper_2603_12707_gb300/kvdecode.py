@@ -240,10 +240,36 @@ def decode_attention_noalloc(k_pool, v_pool, num_pages: int, num_q_heads: int, n
                              head_dim: int, page_table, max_pages: int, lens, q, out,
                              softmax_scale: float = 0.0, device_error=None, stream=None):
     """Allocation-free decode attention over caller-owned pools and page
-    table; ``lens`` is a host sequence of attended token counts, one per row."""
+    table; ``lens`` is a host sequence of attended token counts, one per row.
+
+    Where torch tensors are passed, their dtype, device, layout and shape are
+    checked here before the call, since the kernels read through the raw
+    pointers: page_table int32 [len(lens)][max_pages], q and out bf16
+    [len(lens)][num_q_heads][head_dim], pools bf16 with at least
+    num_pages * num_kv_heads * 16 * head_dim elements, device_error int32."""
     arr = _i32_array(lens)
+    batch = len(arr)
+
+    def _tensor(x, name, dtype, shape=None, min_numel=None):
+        if not hasattr(x, "data_ptr"):
+            return
+        if x.dtype != dtype or not x.is_cuda or not x.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor of {dtype}")
+        if shape is not None and tuple(x.shape) != tuple(shape):
+            raise ValueError(f"{name} must have shape {tuple(shape)}, not {tuple(x.shape)}")
+        if min_numel is not None and x.numel() < min_numel:
+            raise ValueError(f"{name} holds {x.numel()} elements, fewer than {min_numel}")
+
+    import torch
+    _tensor(page_table, "page_table", torch.int32, (batch, max_pages))
+    _tensor(q, "q", torch.bfloat16, (batch, num_q_heads, head_dim))
+    _tensor(out, "out", torch.bfloat16, (batch, num_q_heads, head_dim))
+    pool_elems = int(num_pages) * int(num_kv_heads) * 16 * int(head_dim)
+    _tensor(k_pool, "k_pool", torch.bfloat16, min_numel=pool_elems)
+    _tensor(v_pool, "v_pool", torch.bfloat16, min_numel=pool_elems)
+    _tensor(device_error, "device_error", torch.int32, min_numel=1)
     _check(load().decode_attention_noalloc(_ptr(k_pool), _ptr(v_pool), num_pages, num_q_heads, num_kv_heads,
-                                           head_dim, len(arr), _ptr(page_table), max_pages,
+                                           head_dim, batch, _ptr(page_table), max_pages,
                                            ctypes.addressof(arr), _ptr(q), _ptr(out), float(softmax_scale),
                                            _ptr(device_error), _stream(stream)),
            "decode_attention_noalloc")

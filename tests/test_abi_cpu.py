@@ -243,3 +243,16 @@ def test_split_pages_range(kvlib):
     with pytest.raises(kvlib.KVDecodeError):
         kvlib.kv_cache_set_split_pages(h, 1025)
     kvlib.kv_cache_destroy(h)
+
+
+def test_noalloc_object_references_no_allocator(kvlib):
+    """The entry point's translation unit calls no allocating routine: its
+    object file (built from this repository's source) has no undefined
+    reference to cudaMalloc*, cudaFree*, cuMemAlloc* or cuMemFree*."""
+    import subprocess
+    from paper_2603_12707_gb300 import _build
+    obj = os.path.join(_build.OBJ, "kvd_noalloc.o")
+    r = subprocess.run(["nm", "-u", "-C", obj], capture_output=True, text=True, check=True)
+    bad = [l for l in r.stdout.splitlines()
+           if any(s in l for s in ("cudaMalloc", "cudaFree", "cuMemAlloc", "cuMemFree", "cuMemCreate"))]
+    assert not bad, bad
