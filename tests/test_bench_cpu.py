@@ -100,3 +100,17 @@ def test_clock_records_the_timing_rules_reject():
         assert bench.clocks_slowed({**ok, "reasons": [r]})
     assert bench.clocks_slowed({**ok, "sm_mhz": 1200.0})   # far below max with no reason: a clock lock
     assert not bench.clocks_slowed({"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0})
+
+
+def test_timed_blocks_cover_the_target_time_within_bounds():
+    ns = argparse.Namespace(block_target_s=0.5, min_blocks=3, max_blocks=10)
+    assert bench.block_count(94.0, ns) == 6         # 6 x 94 ms >= 0.5 s
+    assert bench.block_count(11.0, ns) == 10        # capped
+    assert bench.block_count(1080.0, ns) == 3       # at least 3
+    assert bench.block_count(0.0, ns) == 10
+
+
+def test_median_block_is_the_middle_of_the_sorted_times():
+    assert bench.median_block([5.0, 1.0, 3.0]) == 2
+    assert bench.median_block([4.0, 1.0, 3.0, 2.0]) == 3    # lower median: 2.0
+    assert bench.median_block([7.0]) == 0
