@@ -529,16 +529,13 @@ __global__ void __launch_bounds__(kWarps * 32)
         if (pending & (1u << s)) mbar_wait_bounded(smem_addr(&bars[s]), (phase >> s) & 1u, kWaitLimitNs);
     __syncwarp();
 
-    // The last warp out resets the work counter for the next launch.  No
-    // fence: every warp consumed the value of its last counter fetch before
-    // getting here, so all fetches are performed before the reset.
-    if (lane == 0) {
-        const uint32_t total = gridDim.x * kWarps;
-        if (atomicAdd(&p.queue[1], 1u) == total - 1) {
-            p.queue[0] = 0;
-            p.queue[1] = 0;
-        }
-    }
+    // Every warp completes only after the launch it depends on has (so a
+    // launch's completion always implies its predecessor's).  Then one thread
+    // resets the work counter of the next launch: the previous launch used it
+    // and has completed.  The next launch fetches from it only after its own
+    // dependency wait, i.e. after this launch has completed.
+    if (!waited) griddep_wait();
+    if (blockIdx.x == 0 && threadIdx.x == 0 && p.queue_next) *p.queue_next = 0u;
 }
 
 }  // namespace

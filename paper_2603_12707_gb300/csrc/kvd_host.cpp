@@ -92,8 +92,8 @@ struct kv_cache {
     int32_t* meta = nullptr;                    // page table [max_seqs][max_pages], then seq_len [max_seqs]
     int32_t* step_seq = nullptr;
     int2* rows = nullptr;                       // per batch row: (first partial slot, items)
-    uint32_t* queue = nullptr;                  // two (next item, warps done) counter pairs
-    uint32_t fused_launches = 0;                // fused launches alternate counter pairs
+    uint32_t* queue = nullptr;                  // two work counters, used by alternate attention launches
+    uint32_t attn_launches = 0;                 // attention launches so far (selects the counter)
     int64_t launches = 0;                       // kernels launched (reported by kv_cache_query)
     // A fused launch may depend programmatically on the launch before it only
     // if that was an attention launch on the same stream: its early reads
@@ -839,9 +839,11 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.page_stride = c->page_stride;
     p.n_entries_dev = c->step_dev ? c->d_small + 1 : nullptr;
     p.batch = batch;
-    // A fused launch may start while the previous one drains, so consecutive
-    // fused launches use different work counters.
-    p.queue = c->queue + (fused ? 2 * (c->fused_launches & 1u) : 0);
+    // Consecutive attention launches use different work counters: a chained
+    // launch may start while the previous one drains, and each launch resets
+    // the counter of the next one once the previous launch has completed.
+    p.queue = c->queue + (c->attn_launches & 1u);
+    p.queue_next = c->queue + ((c->attn_launches + 1u) & 1u);
     p.err = c->err;
     p.num_pages = c->cfg.num_pages;
     p.n_items = c->step_entries * c->cfg.num_kv_heads;
@@ -871,7 +873,7 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
                               static_cast<cudaStream_t>(stream)));
         ++c->launches;
     }
-    if (fused) ++c->fused_launches;
+    ++c->attn_launches;
     c->chain_launches = c->launches;
     c->chain_stream = stream;
     return KVC_OK;

@@ -177,7 +177,8 @@ struct DecodeParams {
     int32_t page_stride;
     const int32_t* n_entries_dev; // device-built plan: entries live here (n_items is then a bound)
     int32_t batch;
-    uint32_t* queue;          // [0] next item, [1] warps finished
+    uint32_t* queue;          // next item to hand out (zero at launch)
+    uint32_t* queue_next;     // the next launch's counter, reset by this one (null: none)
     int32_t* err;
     int64_t num_pages;
     int32_t n_items;

@@ -58,7 +58,6 @@ __global__ void __launch_bounds__(1024) noalloc_plan_kernel(const __grid_constan
 {
     if (threadIdx.x == 0) {
         a.queue[0] = 0;
-        a.queue[1] = 0;
         if (a.clear_err) *a.err = 0;
     }
     for (int i = threadIdx.x; i < a.batch; i += blockDim.x) {
@@ -257,6 +256,7 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.n_entries_dev = nullptr;
     p.batch = batch;
     p.queue = pa.queue;
+    p.queue_next = nullptr;
     p.err = pa.err;
     p.num_pages = num_pages;
     p.n_items = (int32_t)(entries * num_kv_heads);
