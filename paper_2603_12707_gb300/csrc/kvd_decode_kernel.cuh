@@ -39,6 +39,11 @@ namespace kvd {
 namespace {
 
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
+// Pages of a warp's first item brought into L2 when its dependency wait
+// returns, beyond the ring's stages: the HBM gets new requests at once
+// instead of after the first page's work (Qwen-shaped layers +4 %, the long
+// context +3 %; 1 or 3-4 pages measured no better).
+constexpr int kRampL2Pages = 2;
 constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
 template <int D, bool GQA>
@@ -432,6 +437,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     // griddep_wait() only the plan, page table and cache pages (none of which
     // that kernel writes) are read; q, k_new, v_new and every write come after.
     bool waited = !FUSED;
+    bool first_item = true;
 
     // The first item of every warp is its global warp index; later ones come
     // from the work counter, offset by the number of warps.
@@ -483,6 +489,16 @@ __global__ void __launch_bounds__(kWarps * 32)
             griddep_launch_dependents();
             waited = true;
         }
+        if (first_item && p.kv_map) {
+            // The ring holds this item's first R pages (loaded before the
+            // wait when chained); the next ones go into L2 now.
+            for (int j = R; j < np && j < R + kRampL2Pages; ++j) {
+                int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
+                if (pid < 0 || pid >= p.num_pages) pid = 0;   // recorded when its load is issued
+                if (lane == 0) tma_prefetch_l2_4d(&tmk, 0, (pid * p.H_kv + g) * kPageSize, 0, 0);
+            }
+        }
+        first_item = false;
         comp.start(p, en, g, lane);
 
         for (int j = 0; j < np; ++j) {
