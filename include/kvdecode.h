@@ -114,7 +114,8 @@ KVC_API int kv_cache_destroy(kv_cache *cache);
  * 0 .. num_pages-1, and no page may be in use. */
 KVC_API int kv_cache_set_page_order(kv_cache *cache, const int32_t *order, int64_t n);
 
-/* Synchronise the device and report usage and device error bits.  Returns
+/* Wait for the cache's stream (the stream of its latest call) and report
+ * usage and device error bits.  Returns
  * KVC_ERR_PAGE_TABLE (page or length range), KVC_ERR_OOM (a device-side step
  * ran out of pages) or KVC_ERR_DEVICE (a pipeline wait gave up) if
  * device_error is non-zero; the stats are filled in either way. */
@@ -142,11 +143,19 @@ KVC_API int kv_seq_create(kv_cache *cache, int32_t *seq_id);
  * position is the first slot of a page.  All or nothing: KVC_ERR_OOM if the
  * pool lacks pages, KVC_ERR_INVALID if the row would exceed
  * max_pages_per_seq.  The page-table and length update is enqueued on
- * `stream`. */
+ * `stream`.  While device-side steps are enabled (kv_cache_device_steps) the
+ * device holds the free pages and lengths: the reservation is then one
+ * kernel on `stream`, with no host synchronisation, that takes the same pages
+ * in the same order; a full page row sets KVC_DEVERR_SEQ_RANGE and an
+ * exhausted pool KVC_DEVERR_OOM (read by kv_cache_query) and that
+ * reservation changes nothing; the return code then only covers the
+ * arguments (a live sequence, 0 <= n_tokens <= max_pages_per_seq * 16). */
 KVC_API int kv_seq_reserve(kv_cache *cache, int32_t seq_id, int32_t n_tokens, void *stream);
 
 /* Close a sequence: its pages go back to the front of the pop order in its
- * logical page order.  The device row is reset on `stream`. */
+ * logical page order.  The device row is reset on `stream`.  With device-side
+ * steps enabled this is one kernel on `stream` and no host synchronisation;
+ * the sequence id is free again at once. */
 KVC_API int kv_seq_free(kv_cache *cache, int32_t seq_id, void *stream);
 
 /* Host view of one sequence: *len = reserved positions; page_ids (host,
@@ -158,7 +167,10 @@ KVC_API int kv_seq_info(kv_cache *cache, int32_t seq_id, int32_t *len, int32_t *
 /* Write n tokens of one layer into reserved positions [first_pos,
  * first_pos + n) of a sequence: the prefix (the N_v vision tokens handed over
  * at the modality boundary, then the prompt) or any later rewrite.
- * k, v: device, [n][H_kv][d_h] bf16.  Requires first_pos + n <= length. */
+ * k, v: device, [n][H_kv][d_h] bf16.  Requires first_pos + n <= length:
+ * checked on the host, or, while device-side steps are enabled (the length
+ * is the device's), by the kernel, which then writes nothing and sets
+ * KVC_DEVERR_SEQ_RANGE. */
 KVC_API int kv_write_tokens(kv_cache *cache, int32_t layer, int32_t seq_id, int32_t first_pos,
                     int32_t n, const void *k, const void *v, void *stream);
 
@@ -255,11 +267,16 @@ KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batc
  * replayed every step with no host work (the role CUDA graphs play in the
  * paper's engine, Sec. 5.4).  Enabling reserves plan, page-list and partial
  * buffers for up to max_batch sequences at the longest page-table row, and
- * fixes the work-item size from the pages currently held.  The host
- * allocator's view is refreshed from the device (a device synchronisation)
- * by the next call that needs it: kv_seq_reserve, kv_seq_free, kv_seq_info,
- * kv_begin_step, kv_cache_query, kv_write_tokens, kv_read_tokens,
- * kv_cache_set_page_order, or kv_cache_sync.  Graphs captured while device
+ * fixes the work-item size from the pages currently held.  While enabled,
+ * admitting and closing sequences needs no host synchronisation:
+ * kv_seq_create is host bookkeeping, kv_seq_reserve and kv_seq_free are
+ * kernels on their stream, and kv_write_tokens, kv_write_varlen and
+ * kv_read_tokens check positions against the device's lengths in their
+ * kernels.  The host allocator's view is refreshed from the device lazily,
+ * by the next call that reads it (kv_seq_info, kv_begin_step,
+ * kv_cache_query, kv_cache_set_page_order, kv_cache_device_steps or
+ * kv_cache_sync), which waits for the cache's stream: the stream of the
+ * cache's latest call, so replay the graphs on that stream.  Graphs captured while device
  * steps are enabled stay valid until they are disabled, enabled again (which
  * may resize the buffers) or the cache is destroyed: meanwhile a host-planned
  * step that would need larger buffers fails with KVC_ERR_INVALID instead of
@@ -277,8 +294,8 @@ KVC_API int kv_cache_device_steps(kv_cache *cache, int32_t max_batch, int32_t en
  * host synchronisation; graph-capturable. */
 KVC_API int kv_begin_step_device(kv_cache *cache, int32_t batch, const int32_t *seq_ids, void *stream);
 
-/* Synchronise the device and refresh the host allocator's view after
- * device-side steps. */
+/* Wait for the cache's stream (the stream of its latest call) and refresh the
+ * host allocator's view after device-side steps and allocator calls. */
 KVC_API int kv_cache_sync(kv_cache *cache);
 
 /* ------------------------------------------------ allocation-free decode -- */

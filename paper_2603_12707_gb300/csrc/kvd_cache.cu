@@ -258,9 +258,67 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
     if (threadIdx.x == 0) *a.n_entries = min(entries, a.max_entries);
 }
 
+// Reserve n tokens for a sequence, or release all its pages, on the device
+// free stack, in stream order with device-side steps: a reservation takes
+// the next pages of the stack for the logical pages its new positions open
+// (all or nothing: a full page row sets bit 4, an exhausted pool bit 8, and
+// nothing changes); a release puts the pages back on top of the stack so that
+// its logical page 0 is handed out next, clears its page-table row and sets
+// its length to 0.
+__global__ void __launch_bounds__(256) seq_op_kernel(const SeqOpArgs a)
+{
+    __shared__ int s_len, s_top, s_first, s_count;
+    if (threadIdx.x == 0) {
+        const int len = a.seq_len[a.seq];
+        const int top = *a.free_top;
+        int first = 0, count = 0;
+        if (len < 0 || len > a.max_pages * kPageSize) {
+            flag_error(a.err, 4);
+        } else if (a.free_seq) {
+            count = (len + kPageSize - 1) / kPageSize;
+        } else {
+            const int64_t end = (int64_t)len + a.n;
+            first = (len + kPageSize - 1) / kPageSize;
+            const int64_t need_total = (end + kPageSize - 1) / kPageSize;
+            if (need_total > a.max_pages) {
+                flag_error(a.err, 4);
+            } else if (need_total - first > top) {
+                flag_error(a.err, 8);
+            } else {
+                count = (int)(need_total - first);
+                a.seq_len[a.seq] = (int)end;
+            }
+        }
+        s_len = len;
+        s_top = top;
+        s_first = first;
+        s_count = count;
+    }
+    __syncthreads();
+    int32_t* row = a.page_table + (int64_t)a.seq * a.max_pages;
+    const int top = s_top, first = s_first, count = s_count;
+    if (a.free_seq) {
+        for (int k = threadIdx.x; k < count; k += blockDim.x) {
+            a.free_pages[top + count - 1 - k] = row[k];
+            row[k] = -1;
+        }
+        if (threadIdx.x == 0 && s_len >= 0 && s_len <= a.max_pages * kPageSize) {
+            *a.free_top = top + count;
+            a.seq_len[a.seq] = 0;
+        }
+    } else {
+        for (int k = threadIdx.x; k < count; k += blockDim.x) row[first + k] = a.free_pages[top - 1 - k];
+        if (threadIdx.x == 0) *a.free_top = top - count;
+    }
+}
+
 // One thread per 16-byte chunk of a [n][H_kv][D] token block.
 __global__ void token_copy_kernel(const TokenCopyArgs a)
 {
+    if (a.len && a.first_pos + a.n > *a.len) {   // positions past the sequence's length
+        if (blockIdx.x == 0 && threadIdx.x == 0) flag_error(a.err, 4);
+        return;
+    }
     const int chunks = a.D / 8;
     const int64_t total = (int64_t)a.n * a.H_kv * chunks;
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -309,6 +367,12 @@ __global__ void __launch_bounds__(kVarlenThreads) varlen_write_kernel(const __gr
     const int p0 = max(first, page_idx * kPageSize);
     const int p1 = min(first + a.n_tok[lo], (page_idx + 1) * kPageSize);
     const int nt = p1 - p0;
+    // A block that passes its sequence's length is refused whole (every tile
+    // checks the block's end, not its own).
+    if (a.seq_len && first + a.n_tok[lo] > a.seq_len[a.seq[lo]]) {
+        if (threadIdx.x == 0) flag_error(a.err, 4);
+        return;
+    }
     const int32_t pid = a.page_table[(int64_t)a.seq[lo] * a.max_pages + page_idx];
     if (pid < 0 || pid >= a.num_pages) {
         if (threadIdx.x == 0) flag_error(a.err, 1);
@@ -432,6 +496,12 @@ cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const in
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(want, (int64_t)num_sms * 8));
     gather_pages_kernel<<<grid, 256, 0, st>>>(plan, entries, entries_dev, page_table, max_pages, item_pages,
                                               stride);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_seq_op(const SeqOpArgs& a, cudaStream_t st)
+{
+    seq_op_kernel<<<1, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

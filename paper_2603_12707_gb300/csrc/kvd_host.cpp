@@ -114,6 +114,7 @@ struct kv_cache {
     // device-side steps (kv_begin_step_device): free stack on the device
     bool dev_mode = false;                      // kv_cache_device_steps enabled
     bool dev_dirty = false;                     // the device state moved past the host mirror
+    cudaStream_t last_stream = nullptr;         // stream of the cache's latest enqueued work
     int32_t dev_max_batch = 0;
     int32_t dev_item_pages = 0;
     int32_t dev_entries_cap = 0;
@@ -166,6 +167,7 @@ int push_updates(kv_cache* c, const std::vector<int32_t>& idx, const std::vector
                  cudaStream_t st)
 {
     if (c->host_only || idx.empty()) return KVC_OK;
+    c->last_stream = st;
     ScatterI32 s;
     for (size_t off = 0; off < idx.size(); off += kScatterMax) {
         const size_t n = std::min<size_t>(kScatterMax, idx.size() - off);
@@ -262,21 +264,29 @@ void release_device(kv_cache* c)
     cudaFree(c->part_ml);
 }
 
-// Bring the host mirror up to the device after device-side steps.
+// Bring the host mirror up to the device after device-side steps or
+// allocator calls.  Lazy: only calls that read the mirror (kv_seq_info,
+// kv_cache_query, kv_cache_sync, host-planned steps, page order, enabling or
+// disabling device steps) come here, and they wait for the cache's stream
+// only (the stream of its latest call), not the whole device.
 int sync_from_device(kv_cache* c)
 {
     if (!c->dev_dirty) return KVC_OK;
     const kvc_config& k = c->cfg;
     std::vector<int32_t> pt((size_t)k.max_seqs * k.max_pages_per_seq), lens((size_t)k.max_seqs);
     int32_t small[2] = {0, 0};
-    KVD_CUDA(cudaDeviceSynchronize());
-    KVD_CUDA(cudaMemcpy(pt.data(), c->page_table(), pt.size() * sizeof(int32_t), cudaMemcpyDeviceToHost));
-    KVD_CUDA(cudaMemcpy(lens.data(), c->seq_len_dev(), lens.size() * sizeof(int32_t), cudaMemcpyDeviceToHost));
-    KVD_CUDA(cudaMemcpy(small, c->d_small, sizeof(small), cudaMemcpyDeviceToHost));
+    cudaStream_t st = c->last_stream;
+    KVD_CUDA(cudaMemcpyAsync(pt.data(), c->page_table(), pt.size() * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    KVD_CUDA(cudaMemcpyAsync(lens.data(), c->seq_len_dev(), lens.size() * sizeof(int32_t), cudaMemcpyDeviceToHost,
+                             st));
+    KVD_CUDA(cudaMemcpyAsync(small, c->d_small, sizeof(small), cudaMemcpyDeviceToHost, st));
+    KVD_CUDA(cudaStreamSynchronize(st));
     c->free_stack.assign((size_t)small[0], 0);
-    if (small[0] > 0)
-        KVD_CUDA(cudaMemcpy(c->free_stack.data(), c->d_free, (size_t)small[0] * sizeof(int32_t),
-                            cudaMemcpyDeviceToHost));
+    if (small[0] > 0) {
+        KVD_CUDA(cudaMemcpyAsync(c->free_stack.data(), c->d_free, (size_t)small[0] * sizeof(int32_t),
+                                 cudaMemcpyDeviceToHost, st));
+        KVD_CUDA(cudaStreamSynchronize(st));
+    }
     c->pages_in_use = k.num_pages - small[0];
     for (int32_t s = 0; s < k.max_seqs; ++s) {
         if (c->lens[s] < 0) continue;
@@ -293,6 +303,7 @@ int sync_from_device(kv_cache* c)
 int push_free_stack(kv_cache* c, cudaStream_t st)
 {
     if (!c->dev_mode) return KVC_OK;
+    c->last_stream = st;
     const int32_t top = (int32_t)c->free_stack.size();
     if (top > 0)
         KVD_CUDA(cudaMemcpyAsync(c->d_free, c->free_stack.data(), (size_t)top * sizeof(int32_t),
@@ -439,8 +450,8 @@ int kv_cache_query(kv_cache* c, kvc_stats* s)
     s->device_error = 0;
     s->kernel_launches = c->launches;
     if (c->host_only) return KVC_OK;
-    KVD_CUDA(cudaDeviceSynchronize());
-    KVD_CUDA(cudaMemcpy(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost));
+    KVD_CUDA(cudaMemcpyAsync(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost, c->last_stream));
+    KVD_CUDA(cudaStreamSynchronize(c->last_stream));
     if (s->device_error & (KVC_DEVERR_PAGE_RANGE | KVC_DEVERR_SEQ_RANGE))
         return fail(KVC_ERR_PAGE_TABLE, "device found a page id or length outside its range");
     if (s->device_error & KVC_DEVERR_OOM) return fail(KVC_ERR_OOM, "a device-side step found the page pool exhausted");
@@ -482,9 +493,39 @@ int kv_seq_create(kv_cache* c, int32_t* seq_id)
     return fail(KVC_ERR_OOM, "kv_seq_create: every sequence slot is in use");
 }
 
+// With device-side steps the device holds the free stack, lengths and page
+// table: a reservation or release is a stream-ordered kernel, with no host
+// synchronisation; its failures (full page row, exhausted pool) set device
+// error bits instead of a return code.
+static int seq_op_device(kv_cache* c, int32_t seq, int32_t n, bool free_seq, void* stream)
+{
+    SeqOpArgs a;
+    a.free_seq = free_seq ? 1 : 0;
+    a.seq = seq;
+    a.n = n;
+    a.max_pages = c->cfg.max_pages_per_seq;
+    a.free_pages = c->d_free;
+    a.free_top = c->d_small;
+    a.seq_len = c->seq_len_dev();
+    a.page_table = c->page_table();
+    a.err = c->err;
+    c->last_stream = static_cast<cudaStream_t>(stream);
+    KVD_CUDA(launch_seq_op(a, c->last_stream));
+    ++c->launches;
+    c->dev_dirty = true;
+    return KVC_OK;
+}
+
 int kv_seq_reserve(kv_cache* c, int32_t seq, int32_t n, void* stream)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_seq_reserve: null cache");
+    if (c->dev_mode) {
+        if (int rc = check_seq(c, seq)) return rc;
+        if (n < 0 || (int64_t)n > (int64_t)c->cfg.max_pages_per_seq * kPageSize)
+            return fail(KVC_ERR_INVALID, "kv_seq_reserve: token count outside 0 .. max_pages_per_seq * 16");
+        if (n == 0) return KVC_OK;
+        return seq_op_device(c, seq, n, false, stream);
+    }
     if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     if (n < 0) return fail(KVC_ERR_INVALID, "kv_seq_reserve: negative token count");
@@ -510,6 +551,15 @@ int kv_seq_reserve(kv_cache* c, int32_t seq, int32_t n, void* stream)
 int kv_seq_free(kv_cache* c, int32_t seq, void* stream)
 {
     if (!c) return fail(KVC_ERR_INVALID, "kv_seq_free: null cache");
+    if (c->dev_mode) {
+        if (int rc = check_seq(c, seq)) return rc;
+        if (int rc = seq_op_device(c, seq, 0, true, stream)) return rc;
+        c->lens[seq] = -1;   // the id is free again; its pages and length are the device's
+        c->pages[seq].clear();
+        --c->live;
+        c->step_active = false;
+        return KVC_OK;
+    }
     if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     std::vector<int32_t> idx, val;
@@ -548,10 +598,12 @@ static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq,
 {
     if (!c) return fail(KVC_ERR_INVALID, std::string(what) + ": null cache");
     if (int rc = check_device(c, what)) return rc;
-    if (int rc = sync_from_device(c)) return rc;
     if (int rc = check_seq(c, seq)) return rc;
     if (layer < 0 || layer >= c->cfg.num_layers) return fail(KVC_ERR_INVALID, std::string(what) + ": bad layer");
-    if (first < 0 || n < 0 || (int64_t)first + n > c->lens[seq])
+    // With device-side steps the length lives on the device: the kernel
+    // checks the positions (bit 4 if they pass it); otherwise the host does.
+    const int64_t limit = c->dev_mode ? (int64_t)c->cfg.max_pages_per_seq * kPageSize : c->lens[seq];
+    if (first < 0 || n < 0 || (int64_t)first + n > limit)
         return fail(KVC_ERR_INVALID, std::string(what) + ": positions outside the reserved length");
     if (n == 0) return KVC_OK;
     if (!k || !v || !aligned16(k) || !aligned16(v))
@@ -560,6 +612,7 @@ static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq,
     a.pool_k = c->k_pool(layer);
     a.pool_v = c->v_pool(layer);
     a.pt_row = c->page_table() + (int64_t)seq * c->cfg.max_pages_per_seq;
+    a.len = c->dev_mode ? c->seq_len_dev() + seq : nullptr;
     a.num_pages = c->cfg.num_pages;
     a.H_kv = c->cfg.num_kv_heads;
     a.D = c->cfg.head_dim;
@@ -569,6 +622,7 @@ static int token_copy(kv_cache* c, const char* what, int32_t layer, int32_t seq,
     a.tok_v = static_cast<uint16_t*>(v);
     a.to_pool = to_pool;
     a.err = c->err;
+    c->last_stream = static_cast<cudaStream_t>(stream);
     KVD_CUDA(launch_token_copy(a, static_cast<cudaStream_t>(stream)));
     ++c->launches;
     return KVC_OK;
@@ -592,7 +646,6 @@ int kv_write_varlen(kv_cache* c, int32_t layer_first, int32_t n_layers, int32_t 
 {
     if (!c || (n_blocks > 0 && (!seq_ids || !cu_seqlens)))
         return fail(KVC_ERR_INVALID, "kv_write_varlen: null argument");
-    if (int rc = sync_from_device(c)) return rc;
     if (n_layers < 1 || n_layers > 65535 || layer_first < 0 || (int64_t)layer_first + n_layers > c->cfg.num_layers)
         return fail(KVC_ERR_INVALID, "kv_write_varlen: layers outside the cache");
     if (n_blocks < 0) return fail(KVC_ERR_INVALID, "kv_write_varlen: negative block count");
@@ -604,7 +657,9 @@ int kv_write_varlen(kv_cache* c, int32_t layer_first, int32_t n_layers, int32_t 
         const int64_t n = (int64_t)cu_seqlens[i + 1] - cu_seqlens[i];
         const int64_t f = first_pos ? first_pos[i] : 0;
         if (n < 0) return fail(KVC_ERR_INVALID, "kv_write_varlen: cu_seqlens must not decrease");
-        if (f < 0 || f + n > c->lens[seq_ids[i]])
+        // with device-side steps the kernel checks against the device's length
+        const int64_t limit = c->dev_mode ? (int64_t)c->cfg.max_pages_per_seq * kPageSize : c->lens[seq_ids[i]];
+        if (f < 0 || f + n > limit)
             return fail(KVC_ERR_INVALID, "kv_write_varlen: positions outside the reserved length");
         order[i] = i;
     }
@@ -636,12 +691,14 @@ int kv_write_varlen(kv_cache* c, int32_t layer_first, int32_t n_layers, int32_t 
     a.v = static_cast<const uint16_t*>(v);
     a.src_layer_stride = rows * c->cfg.num_kv_heads * c->cfg.head_dim;
     a.page_table = c->page_table();
+    a.seq_len = c->dev_mode ? c->seq_len_dev() : nullptr;
     a.num_pages = c->cfg.num_pages;
     a.max_pages = c->cfg.max_pages_per_seq;
     a.H_kv = c->cfg.num_kv_heads;
     a.D = c->cfg.head_dim;
     a.err = c->err;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    c->last_stream = st;
     // Blocks go kVarlenMax at a time (empty ones skipped), one launch each.
     auto flush = [&]() -> int {
         if (a.n_blocks == 0) return KVC_OK;
@@ -737,6 +794,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     c->step_active = false;
     if (!c->host_only) {
         cudaStream_t st = static_cast<cudaStream_t>(stream);
+        c->last_stream = st;
         StepPatch patch;
         PlanArgs pa;
         pa.batch = batch;
@@ -810,6 +868,7 @@ int kv_append(kv_cache* c, int32_t layer, int32_t batch, const void* k_new, cons
     a.D = c->cfg.head_dim;
     a.max_pages = c->cfg.max_pages_per_seq;
     a.err = c->err;
+    c->last_stream = static_cast<cudaStream_t>(stream);
     KVD_CUDA(launch_append(a, static_cast<cudaStream_t>(stream)));
     ++c->launches;
     return KVC_OK;
@@ -861,6 +920,7 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
     p.kv_map = 1;
     const bool pdl = fused && c->chain_launches == c->launches && c->chain_stream == stream;
+    c->last_stream = static_cast<cudaStream_t>(stream);
     KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, pdl, grid, c->tmaps[layer], c->tmaps[layer], p,
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
@@ -952,6 +1012,7 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     a.page_ids = c->item_pages;
     a.page_stride = c->dev_stride;
     a.err = c->err;
+    c->last_stream = st;
     KVD_CUDA(launch_step_device(a, st));
     ++c->launches;
     c->dev_dirty = true;

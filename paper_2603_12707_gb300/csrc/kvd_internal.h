@@ -115,10 +115,24 @@ struct ScatterI32 {
     int32_t val[kScatterMax];
 };
 
+// Sequence reservation or release on the device free stack (device-side
+// steps enabled): the same pages, in the same order, as the host allocator.
+struct SeqOpArgs {
+    int32_t free_seq;         // 0: reserve n tokens, 1: release every page of the sequence
+    int32_t seq, n;
+    int32_t max_pages;        // page-table row length
+    int32_t* free_pages;      // device free stack; the next page is free_pages[*free_top - 1]
+    int32_t* free_top;
+    int32_t* seq_len;
+    int32_t* page_table;
+    int32_t* err;
+};
+
 struct TokenCopyArgs {
     uint16_t* pool_k;         // layer pool base [num_pages][H_kv][P][D]
     uint16_t* pool_v;
     const int32_t* pt_row;    // page-table row of the sequence (device)
+    const int32_t* len;       // the sequence's length (device), or null: positions checked on the host
     int64_t num_pages;
     int32_t H_kv, D;
     int32_t first_pos, n;
@@ -140,6 +154,7 @@ struct VarlenWriteArgs {
     const uint16_t* v;
     int64_t src_layer_stride;    // rows * H_kv * D
     const int32_t* page_table;   // [max_seqs][max_pages]
+    const int32_t* seq_len;      // [max_seqs] (device), or null: positions checked on the host
     int64_t num_pages;
     int32_t max_pages;
     int32_t H_kv, D;
@@ -219,6 +234,7 @@ cudaError_t launch_gather_pages(const PlanEntry* plan, int32_t entries, const in
                                 const int32_t* page_table, int32_t max_pages, int32_t* item_pages, int32_t stride,
                                 int num_sms, cudaStream_t st);
 cudaError_t launch_step_device(const StepDevArgs& a, cudaStream_t st);
+cudaError_t launch_seq_op(const SeqOpArgs& a, cudaStream_t st);
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
 cudaError_t launch_wait_timeout_check(uint64_t limit_ns, int32_t* status, cudaStream_t st);
 
