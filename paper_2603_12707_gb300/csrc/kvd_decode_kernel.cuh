@@ -20,6 +20,14 @@
 // Q.K^T and P.V as m16n8k16 bf16 MMAs with the 16 tokens of a page as M and the
 // G heads (padded to 8) as N.
 //
+// Chained launches (programmatic dependent launch, decode_attention_append
+// after another attention launch): a warp issues its first item's ring loads
+// before the dependency wait, and right after it brings the item's next
+// kRampL2Pages pages into L2, so the HBM keeps streaming while the ring's
+// pages are worked.  Consecutive launches use alternating work counters; each
+// launch resets the next one's after its wait, so no warp does an atomic on
+// its way out.
+//
 // Every mbarrier wait is bounded: after a second without progress the warp
 // records KVC_DEVERR_WAIT_TIMEOUT, waits (bounded) for its loads in flight and
 // leaves.  Page ids outside the pool are recorded and replaced by page 0.
