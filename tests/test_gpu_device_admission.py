@@ -2,10 +2,10 @@
 CUDA graph, with no host synchronisation (lazy allocation at prefill entry,
 Sec. 5.4 "Lazy KV Cache Allocation").
 
-One stream carries everything: a bounded GPU sleep first, then replayed decode
+One stream carries everything: a bounded GPU wait first, then replayed decode
 steps interleaved with sequence frees, creations, prompt reservations, packed
 prefix writes and the batch's id swaps.  The event recorded right after the
-sleep must still be pending once the last call has returned: no call waited
+wait must still be pending once the last call has returned: no call waited
 for the GPU.  Afterwards the page tables equal the allocator model's for the
 same calls, every output of the last step matches the float64 oracle, and the
 device error word is clear.  Failures on the device path (an exhausted pool,
@@ -97,10 +97,13 @@ def test_admissions_and_frees_between_replayed_steps_need_no_host_sync(kvlib, Hq
     swaps = [torch.empty(B, dtype=torch.int32).pin_memory() for _ in range(3)]
     stream.synchronize()
 
-    # ---- the window: nothing below may wait for the GPU
+    # ---- the window: nothing below may wait for the GPU.  The stream is held
+    # first by the library's bounded wait diagnostic (a 0.3 s wait on a
+    # barrier nothing completes, which then records that it gave up).
     after_sleep = torch.cuda.Event()
+    waited = torch.zeros(1, dtype=torch.int32, device="cuda")
     with torch.cuda.stream(stream):
-        torch.cuda._sleep(int(4e8))                       # bounded spin, ~0.2 s at 2 GHz
+        kd.kv_selftest_wait_timeout(300_000_000, waited, stream)
         after_sleep.record(stream)
         t0 = time.perf_counter()
         for reps, slot in ((2, 1), (3, 3), (1, 0)):
@@ -120,8 +123,9 @@ def test_admissions_and_frees_between_replayed_steps_need_no_host_sync(kvlib, Hq
             stepped(batch)
         host_s = time.perf_counter() - t0
         pending = not after_sleep.query()
-    assert pending, f"a call waited for the GPU (the sleep had finished after {host_s:.3f} s of host calls)"
+    assert pending, f"a call waited for the GPU (the wait had ended after {host_s:.3f} s of host calls)"
     stream.synchronize()
+    assert int(waited.item()) == 1
 
     # ---- the state and the last step's outputs
     st = kd.kv_cache_query(h)
