@@ -114,3 +114,48 @@ def test_median_block_is_the_middle_of_the_sorted_times():
     assert bench.median_block([5.0, 1.0, 3.0]) == 2
     assert bench.median_block([4.0, 1.0, 3.0, 2.0]) == 3    # lower median: 2.0
     assert bench.median_block([7.0]) == 0
+
+
+def _fake_run(cfg, block_ms, steps, L):
+    """A run record as run_gpu returns it: blocks of `steps` steps whose
+    attended lengths grow by one per step."""
+    blocks = []
+    lens = [100, 200]
+    for ms in block_ms:
+        step_bytes, attn_bytes = [], []
+        for _ in range(steps):
+            att = [n + 1 for n in lens]
+            a, p = bench.layer_bytes(cfg, att)
+            step_bytes.append(L * (a + p))
+            attn_bytes.append(a + p)
+            lens = [n + 1 for n in lens]
+        blocks.append({"ms": ms, "step_ms": [ms / steps] * steps, "attn_ms": [0.9 * ms / steps / L] * steps,
+                       "step_bytes": step_bytes, "attn_bytes": attn_bytes})
+    clocks = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 12, "retimed": False}
+    e2e = {"ms": 1.1 * sum(block_ms) / len(block_ms), "wall_s": 0.1, "bytes": sum(blocks[0]["step_bytes"]),
+           "h2d": 1000, "d2h": 500}
+    return {"blocks": blocks, "launches": 3 * steps, "clocks": clocks, "e2e": e2e, "cfg": cfg, "L": L}
+
+
+def test_summary_reports_the_median_block_and_every_contract_key():
+    import dataclasses
+    cfg = dataclasses.replace(wl.custom("fake", 2, 8, 8, 64, 2, lens=[100, 200], seed=1), phys_layers=2)
+    steps, L = 4, 2
+    ns = argparse.Namespace(steps=steps, config="tiny", page_order=None, unfused=False, split_pages=0, graph=True)
+    r = _fake_run(cfg, [3.0, 1.0, 2.0], steps, L)
+    out = bench.summarize(ns, 1, r)
+    mid = r["blocks"][2]                       # 2.0 ms is the median of 3.0, 1.0, 2.0
+    assert out["ms_per_step"] == round(2.0 / steps, 4)
+    assert out["value"] == round(sum(mid["step_bytes"]) / 2.0e-3 / 1e9, 2)
+    assert out["steps_per_s"] == round(steps / 2.0e-3, 3)
+    assert out["timed_blocks"] == 3 and out["block_ms"] == [3.0, 1.0, 2.0]
+    all_gbs = sum(sum(b["step_bytes"]) for b in r["blocks"]) / 6.0e-3 / 1e9
+    assert out["all_blocks_gbs"] == round(all_gbs, 2)
+    ro = out["roofline"]
+    assert set(ro) >= {"bound", "achieved", "peak", "unit", "frac", "traffic"}
+    assert ro["bound"] == "hbm" and ro["unit"] == "GB/s"
+    assert abs(ro["frac"] - ro["achieved"] / ro["peak"]) < 1e-3
+    assert out["e2e"]["h2d_bytes_per_step"] == 1000 and out["e2e"]["d2h_bytes_per_step"] == 500
+    assert out["e2e"]["unit"] == "GB/s" and out["e2e"]["value"] > 0
+    assert out["clocks"]["samples"] == 12 and out["gpu_launches"] == 3 * steps
+    assert out["config"]["workload"].startswith("fake") and "l2" in out["config"]
