@@ -115,6 +115,7 @@ struct kv_cache {
     bool dev_mode = false;                      // kv_cache_device_steps enabled
     bool dev_dirty = false;                     // the device state moved past the host mirror
     cudaStream_t last_stream = nullptr;         // stream of the cache's latest enqueued work
+    cudaStream_t copy_stream = nullptr;         // the cache's own stream for reading its state back
     int32_t dev_max_batch = 0;
     int32_t dev_item_pages = 0;
     int32_t dev_entries_cap = 0;
@@ -250,6 +251,7 @@ int grow_scratch(kv_cache* c, int64_t entries, int64_t slots, int64_t page_ids, 
 
 void release_device(kv_cache* c)
 {
+    if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
     cudaFree(c->pools);
     cudaFree(c->meta);
     cudaFree(c->step_seq);
@@ -264,18 +266,32 @@ void release_device(kv_cache* c)
     cudaFree(c->part_ml);
 }
 
+// Wait for the cache's stream (the stream of its latest call).  Should that
+// handle no longer be a stream (the caller destroyed it), wait for the device.
+int wait_cache_stream(kv_cache* c)
+{
+    if (cudaStreamSynchronize(c->last_stream) != cudaSuccess) {
+        cudaGetLastError();
+        c->last_stream = nullptr;
+        KVD_CUDA(cudaDeviceSynchronize());
+    }
+    return KVC_OK;
+}
+
 // Bring the host mirror up to the device after device-side steps or
 // allocator calls.  Lazy: only calls that read the mirror (kv_seq_info,
 // kv_cache_query, kv_cache_sync, host-planned steps, page order, enabling or
 // disabling device steps) come here, and they wait for the cache's stream
-// only (the stream of its latest call), not the whole device.
+// only, not the whole device; the state is then read back on the cache's own
+// stream.
 int sync_from_device(kv_cache* c)
 {
     if (!c->dev_dirty) return KVC_OK;
     const kvc_config& k = c->cfg;
     std::vector<int32_t> pt((size_t)k.max_seqs * k.max_pages_per_seq), lens((size_t)k.max_seqs);
     int32_t small[2] = {0, 0};
-    cudaStream_t st = c->last_stream;
+    if (int rc = wait_cache_stream(c)) return rc;
+    cudaStream_t st = c->copy_stream;
     KVD_CUDA(cudaMemcpyAsync(pt.data(), c->page_table(), pt.size() * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
     KVD_CUDA(cudaMemcpyAsync(lens.data(), c->seq_len_dev(), lens.size() * sizeof(int32_t), cudaMemcpyDeviceToHost,
                              st));
@@ -366,6 +382,8 @@ int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
                              std::string(#call) + ": " + cudaGetErrorString(e_)));         \
     } while (0)
         KVD_CUDA_C(cudaGetDevice(&c->device));
+        KVD_CUDA_C(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+        c->last_stream = st;
         KVD_CUDA_C(cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device));
         KVD_CUDA_C(decode_variant_info(k.head_dim, c->group > 1, &c->variant));
         auto encode = tensor_map_encoder();
@@ -450,8 +468,9 @@ int kv_cache_query(kv_cache* c, kvc_stats* s)
     s->device_error = 0;
     s->kernel_launches = c->launches;
     if (c->host_only) return KVC_OK;
-    KVD_CUDA(cudaMemcpyAsync(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost, c->last_stream));
-    KVD_CUDA(cudaStreamSynchronize(c->last_stream));
+    if (int rc = wait_cache_stream(c)) return rc;
+    KVD_CUDA(cudaMemcpyAsync(&s->device_error, c->err, sizeof(int32_t), cudaMemcpyDeviceToHost, c->copy_stream));
+    KVD_CUDA(cudaStreamSynchronize(c->copy_stream));
     if (s->device_error & (KVC_DEVERR_PAGE_RANGE | KVC_DEVERR_SEQ_RANGE))
         return fail(KVC_ERR_PAGE_TABLE, "device found a page id or length outside its range");
     if (s->device_error & KVC_DEVERR_OOM) return fail(KVC_ERR_OOM, "a device-side step found the page pool exhausted");
