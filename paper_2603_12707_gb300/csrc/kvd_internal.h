@@ -37,7 +37,8 @@ struct PlanEntry {
 // items and the warps run out of work at nearly the same time.
 __host__ __device__ inline int row_item_pages(int T, int i, int n)
 {
-    if (10 * (int64_t)i >= 9 * (int64_t)n) return T >= 4 ? T / 4 : 1;
+    if (100 * (int64_t)i >= 95 * (int64_t)n) return T >= 8 ? T / 8 : 1;
+    if (100 * (int64_t)i >= 85 * (int64_t)n) return T >= 4 ? T / 4 : 1;
     if (10 * (int64_t)i >= 7 * (int64_t)n) return T >= 2 ? T / 2 : 1;
     return T;
 }
