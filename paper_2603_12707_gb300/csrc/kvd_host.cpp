@@ -943,6 +943,7 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, pdl, grid, c->tmaps[layer], c->tmaps[layer], p,
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
+    ++c->attn_launches;   // the launch used one counter and resets the other, whatever follows
     if (c->step_split) {
         // Launched early (fused), the merge CTAs sit beside the resident split pass.
         const int split_regs =
@@ -952,7 +953,6 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
                               static_cast<cudaStream_t>(stream)));
         ++c->launches;
     }
-    ++c->attn_launches;
     c->chain_launches = c->launches;
     c->chain_stream = stream;
     return KVC_OK;
