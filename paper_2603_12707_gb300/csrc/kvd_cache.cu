@@ -159,6 +159,7 @@ __global__ void __launch_bounds__(1024)
             }
         },
         a.plan, a.rows, a.page_table, a.max_pages, a.page_ids, a.page_stride, a.err);
+    if (threadIdx.x == 0) *a.step_no += 1u;
 }
 
 // The same step on the device (graph-replayable, no host input): rows in
@@ -255,7 +256,10 @@ __global__ void __launch_bounds__(1024) step_device_kernel(const StepDevArgs a)
             if (*seq < 0) *seq = 0;
         },
         a.plan, a.rows, a.page_table, a.max_pages, a.page_ids, a.page_stride, a.err);
-    if (threadIdx.x == 0) *a.n_entries = min(entries, a.max_entries);
+    if (threadIdx.x == 0) {
+        *a.n_entries = min(entries, a.max_entries);
+        *a.step_no += 1u;
+    }
 }
 
 // Reserve n tokens for a sequence, or release all its pages, on the device

@@ -22,9 +22,11 @@
 //
 // Chained launches (programmatic dependent launch, decode_attention_append
 // after another attention launch): a warp issues its first item's ring loads
-// before the dependency wait, and right after it brings the item's next
-// kRampL2Pages pages into L2, so the HBM keeps streaming while the ring's
-// pages are worked.  Consecutive launches use alternating work counters; each
+// before the dependency wait; once the previous launch's merge pass announces
+// (start_flags) that its split pass is complete, the warp brings the item's
+// next kEarlyL2Pages pages into L2; and right after its wait it brings the
+// next kRampL2Pages, so the HBM keeps streaming while the merge runs and the
+// ring's pages are worked.  Consecutive launches use alternating work counters; each
 // launch resets the next one's after its wait, so no warp does an atomic on
 // its way out.
 //
@@ -52,6 +54,14 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;
 // instead of after the first page's work (Qwen-shaped layers +4 %, the long
 // context +3 %; 1 or 3-4 pages measured no better).
 constexpr int kRampL2Pages = 2;
+// Pages brought into L2 earlier still, once the previous launch's merge pass
+// has announced that its split pass is complete (while that merge runs):
+// +0.4 % per step on the LLaVA and Qwen shapes; 2-3 pages cost the Qwen shape.
+constexpr int kEarlyL2Pages = 1;
+// How long a warp waits for that announcement at most (it comes within
+// microseconds when the launches are chained; the dependency wait follows in
+// any case).
+constexpr uint64_t kEarlyPollLimitNs = 2000000ull;
 constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
 template <int D, bool GQA>
@@ -492,6 +502,28 @@ __global__ void __launch_bounds__(kWarps * 32)
         __syncwarp();
         for (int j = 0; j < pre; ++j) issue(j, j);
         pending = (1u << pre) - 1u;
+        int ramp0 = R;   // first page of the L2 ramp at the wait's return
+        if (!waited && p.prev_tag && np > R && p.kv_map) {
+            unsigned smid;
+            asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+            const uint32_t want = *p.step_no * 65536u + p.prev_tag;
+            const volatile uint32_t* flag = p.start_flags + (smid % (unsigned)p.num_sms) * 32;
+            const uint64_t t0 = global_timer_ns();
+            bool seen = false;
+            while (true) {
+                seen = *flag == want;
+                if (seen || global_timer_ns() - t0 > kEarlyPollLimitNs) break;
+                __nanosleep(128);
+            }
+            if (seen) {
+                for (int j = R; j < np && j < R + kEarlyL2Pages; ++j) {
+                    int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
+                    if (pid < 0 || pid >= p.num_pages) pid = 0;   // recorded when its load is issued
+                    if (lane == 0) tma_prefetch_l2_4d(&tmk, 0, (pid * p.H_kv + g) * kPageSize, 0, 0);
+                }
+                ramp0 = R + kEarlyL2Pages;
+            }
+        }
         if (!waited) {
             griddep_wait();
             griddep_launch_dependents();
@@ -500,7 +532,7 @@ __global__ void __launch_bounds__(kWarps * 32)
         if (first_item && p.kv_map) {
             // The ring holds this item's first R pages (loaded before the
             // wait when chained); the next ones go into L2 now.
-            for (int j = R; j < np && j < R + kRampL2Pages; ++j) {
+            for (int j = ramp0; j < np && j < ramp0 + kRampL2Pages; ++j) {
                 int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
                 if (pid < 0 || pid >= p.num_pages) pid = 0;   // recorded when its load is issued
                 if (lane == 0) tma_prefetch_l2_4d(&tmk, 0, (pid * p.H_kv + g) * kPageSize, 0, 0);

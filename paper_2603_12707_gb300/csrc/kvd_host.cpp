@@ -93,6 +93,10 @@ struct kv_cache {
     int32_t* step_seq = nullptr;
     int2* rows = nullptr;                       // per batch row: (first partial slot, items)
     uint32_t* queue = nullptr;                  // two work counters, used by alternate attention launches
+    uint32_t* start_flags = nullptr;            // [num_sms][32]: merge passes announce their split pass's end
+    uint32_t* step_no = nullptr;                // device step counter
+    uint32_t attn_tag = 0;                      // tag of the step's latest attention launch (0: none yet)
+    bool prev_merge = false;                    // that launch has a merge pass
     uint32_t attn_launches = 0;                 // attention launches so far (selects the counter)
     int64_t launches = 0;                       // kernels launched (reported by kv_cache_query)
     // A fused launch may depend programmatically on the launch before it only
@@ -257,6 +261,8 @@ void release_device(kv_cache* c)
     cudaFree(c->step_seq);
     cudaFree(c->rows);
     cudaFree(c->queue);
+    cudaFree(c->start_flags);
+    cudaFree(c->step_no);
     cudaFree(c->err);
     cudaFree(c->plan);
     cudaFree(c->item_pages);
@@ -397,6 +403,10 @@ int kv_cache_create(const kvc_config* cfg, void* stream, kv_cache** out)
         KVD_CUDA_C(cudaMalloc((void**)&c->step_seq, (size_t)k.max_seqs * sizeof(int32_t)));
         KVD_CUDA_C(cudaMalloc((void**)&c->rows, (size_t)k.max_seqs * sizeof(int2)));
         KVD_CUDA_C(cudaMalloc((void**)&c->queue, 4 * sizeof(uint32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->start_flags, (size_t)c->num_sms * 32 * sizeof(uint32_t)));
+        KVD_CUDA_C(cudaMalloc((void**)&c->step_no, sizeof(uint32_t)));
+        KVD_CUDA_C(cudaMemsetAsync(c->start_flags, 0, (size_t)c->num_sms * 32 * sizeof(uint32_t), st));
+        KVD_CUDA_C(cudaMemsetAsync(c->step_no, 0, sizeof(uint32_t), st));
         KVD_CUDA_C(cudaMalloc((void**)&c->err, sizeof(int32_t)));
         KVD_CUDA_C(cudaMemsetAsync(c->pools, 0, pool_bytes, st));
         KVD_CUDA_C(cudaMemsetAsync(c->meta, 0xff, (size_t)k.max_seqs * k.max_pages_per_seq * sizeof(int32_t), st));
@@ -828,6 +838,7 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
         pa.page_ids = c->item_pages;
         pa.page_stride = stride;
         pa.err = c->err;
+        pa.step_no = c->step_no;
         // Longest rows first: their items start early and the tail is short.
         pa.use_order = use_order ? 1 : 0;
         if (use_order)
@@ -848,6 +859,8 @@ int kv_begin_step(kv_cache* c, int32_t batch, const int32_t* seq_ids, void* stre
     }
     if (!c->host_only)
         if (int rc = push_free_stack(c, static_cast<cudaStream_t>(stream))) return rc;
+    c->attn_tag = 0;
+    c->prev_merge = false;
     c->step_active = true;
     c->step_dev = false;
     c->step_split = split;
@@ -939,11 +952,19 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     const int grid = (int)std::max<int64_t>(1, std::min(resident, want));
     p.kv_map = 1;
     const bool pdl = fused && c->chain_launches == c->launches && c->chain_stream == stream;
+    // The early L2 start waits for the previous launch's merge pass, so only
+    // a launch chained after one that has a merge pass looks for it.
+    p.start_flags = c->start_flags;
+    p.step_no = c->step_no;
+    p.prev_tag = (pdl && c->prev_merge) ? c->attn_tag : 0;
+    p.tag = ++c->attn_tag;
+    p.num_sms = c->num_sms;
     c->last_stream = static_cast<cudaStream_t>(stream);
     KVD_CUDA(launch_decode(c->cfg.head_dim, c->group > 1, fused, pdl, grid, c->tmaps[layer], c->tmaps[layer], p,
                            static_cast<cudaStream_t>(stream)));
     ++c->launches;
     ++c->attn_launches;   // the launch used one counter and resets the other, whatever follows
+    c->prev_merge = false;
     if (c->step_split) {
         // Launched early (fused), the merge CTAs sit beside the resident split pass.
         const int split_regs =
@@ -952,6 +973,7 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
         KVD_CUDA(launch_merge(c->cfg.head_dim, fused, c->step_max_chunks, c->num_sms, split_regs, p,
                               static_cast<cudaStream_t>(stream)));
         ++c->launches;
+        c->prev_merge = true;
     }
     c->chain_launches = c->launches;
     c->chain_stream = stream;
@@ -1031,10 +1053,13 @@ int kv_begin_step_device(kv_cache* c, int32_t batch, const int32_t* seq_ids, voi
     a.page_ids = c->item_pages;
     a.page_stride = c->dev_stride;
     a.err = c->err;
+    a.step_no = c->step_no;
     c->last_stream = st;
     KVD_CUDA(launch_step_device(a, st));
     ++c->launches;
     c->dev_dirty = true;
+    c->attn_tag = 0;
+    c->prev_merge = false;
     c->step_active = true;
     c->step_dev = true;
     c->step_split = true;   // the row split is only known on the device: always run the merge pass

@@ -86,6 +86,7 @@ struct PlanArgs {
     int32_t* page_ids;   // [entries][page_stride]: page ids of each entry's pages
     int32_t page_stride;
     int32_t* err;
+    uint32_t* step_no;   // step counter, advanced by the launch that builds the plan
 };
 
 // kv_begin_step_device: the step's lazy allocation and plan, on the device.
@@ -108,6 +109,7 @@ struct StepDevArgs {
     int32_t* page_ids;        // [max_entries][page_stride]: page ids of each entry's pages
     int32_t page_stride;
     int32_t* err;
+    uint32_t* step_no;        // step counter, advanced once per step
 };
 
 struct ScatterI32 {
@@ -210,6 +212,17 @@ struct DecodeParams {
     // 1: the first tensor map covers K and V (one 4-D load per page); 0: two
     // 3-D maps, K and V.
     int32_t kv_map;
+    // Early start of a chained launch: the merge pass of each launch writes
+    // step * 65536 + tag into every SM's word of start_flags (one word per
+    // 128-byte line) once its dependency wait has returned, i.e. once that
+    // launch's split pass is complete; a launch with prev_tag != 0 (chained
+    // after a launch that has a merge pass) waits for its predecessor's value
+    // before its own dependency wait and then brings more of its first item
+    // into L2.  step_no is the device step counter (the step kernels count).
+    uint32_t* start_flags;
+    const uint32_t* step_no;
+    uint32_t tag, prev_tag;
+    int32_t num_sms;
 };
 
 // TMA view of a (page, head) tile: box {64 columns, 16 rows, D/64 column

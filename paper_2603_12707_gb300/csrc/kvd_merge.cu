@@ -124,6 +124,12 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
         griddep_launch_dependents();   // the next layer may start streaming now
         griddep_wait();                // the split pass of this layer is complete
     }
+    // Announce that the split pass is complete to the next layer's warps,
+    // which are resident already and warm L2 while this pass runs.
+    if (blockIdx.x == 0 && p.start_flags) {
+        const uint32_t v = *p.step_no * 65536u + p.tag;
+        for (int k = lane; k < p.num_sms; k += 32) p.start_flags[k * 32] = v;
+    }
     for (bool first = true; w < total; w += gridDim.x * kMergeWarps, first = false) {
         const int part = w % kMergeSplit;
         const int bh = w / kMergeSplit;

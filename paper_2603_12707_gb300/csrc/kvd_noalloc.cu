@@ -266,6 +266,10 @@ extern "C" KVC_API int decode_attention_noalloc(const void* k_pool, const void* 
     p.max_pages = max_pages;
     p.scale_log2 = scale * 1.4426950408889634f;
     p.kv_map = 0;
+    p.start_flags = nullptr;
+    p.step_no = nullptr;
+    p.tag = p.prev_tag = 0;
+    p.num_sms = num_sms;
     p.k_new = p.v_new = nullptr;
     p.pool_k = p.pool_v = nullptr;
     const int64_t resident = (int64_t)num_sms * std::max(1, var.ctas_per_sm);
