@@ -58,10 +58,10 @@ constexpr int kRampL2Pages = 2;
 // has announced that its split pass is complete (while that merge runs):
 // +0.4 % per step on the LLaVA and Qwen shapes; 2-3 pages cost the Qwen shape.
 constexpr int kEarlyL2Pages = 1;
-// How long a warp waits for that announcement at most (it comes within
-// microseconds when the launches are chained; the dependency wait follows in
-// any case).
-constexpr uint64_t kEarlyPollLimitNs = 2000000ull;
+// How long a warp waits for that announcement at most (it comes once the
+// previous split pass has ended, which chained CTAs see from its tail; the
+// dependency wait follows in any case).
+constexpr uint64_t kEarlyPollLimitNs = 500000ull;
 constexpr int kWarps = 1;   // one warp per CTA: a CTA's resources free up as soon as its warp is done
 
 template <int D, bool GQA>

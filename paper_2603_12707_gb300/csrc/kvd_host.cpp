@@ -97,6 +97,7 @@ struct kv_cache {
     uint32_t* step_no = nullptr;                // device step counter
     uint32_t attn_tag = 0;                      // tag of the step's latest attention launch (0: none yet)
     bool prev_merge = false;                    // that launch has a merge pass
+    unsigned long long prev_capture = 0;        // its stream-capture sequence (0: not captured)
     uint32_t attn_launches = 0;                 // attention launches so far (selects the counter)
     int64_t launches = 0;                       // kernels launched (reported by kv_cache_query)
     // A fused launch may depend programmatically on the launch before it only
@@ -953,10 +954,22 @@ static int launch_attention(kv_cache* c, const char* what, int32_t layer, int32_
     p.kv_map = 1;
     const bool pdl = fused && c->chain_launches == c->launches && c->chain_stream == stream;
     // The early L2 start waits for the previous launch's merge pass, so only
-    // a launch chained after one that has a merge pass looks for it.
+    // a launch chained after one that has a merge pass looks for it, and only
+    // when both were issued the same way: eagerly, or into the same stream
+    // capture (a graph replays its own launches in order, but what precedes
+    // a graph's first launch at replay is not what preceded it at capture).
+    unsigned long long capture = 0;
+    {
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamGetCaptureInfo(static_cast<cudaStream_t>(stream), &cs, &capture) != cudaSuccess ||
+            cs != cudaStreamCaptureStatusActive)
+            capture = 0;
+        cudaGetLastError();
+    }
     p.start_flags = c->start_flags;
     p.step_no = c->step_no;
-    p.prev_tag = (pdl && c->prev_merge) ? c->attn_tag : 0;
+    p.prev_tag = (pdl && c->prev_merge && capture == c->prev_capture) ? c->attn_tag : 0;
+    c->prev_capture = capture;
     p.tag = ++c->attn_tag;
     p.num_sms = c->num_sms;
     c->last_stream = static_cast<cudaStream_t>(stream);

@@ -280,3 +280,56 @@ def test_batch_beyond_one_block_device_and_host_steps(kvlib):
         assert_close(bf16_to_f64(ob)[keep], ref, vmax, gqa=True, what=step)
     a.close()
     b.close()
+
+
+def test_layer_graph_captured_after_another_replays_as_fast(kvlib):
+    """Two graphs of the same fused layers, captured one after the other, each
+    replayed after a graph of the device-side step: the second graph's first
+    layer must not wait for an announcement from the first graph's last
+    layer, which at replay is not its predecessor (its time stays within 2x
+    of the first graph's; a missed announcement would add its 0.5 ms wait)."""
+    cfg = wl.custom("twographs", 4, 8, 8, 64, 4, lens=[300, 17, 900, 64], seed=21)
+    t = Tracked(cfg, keep_host=False, extra_tokens=200)
+    h = t.sess.h
+    B, L = cfg.batch, cfg.num_layers
+    stream = torch.cuda.Stream()
+    ids = torch.tensor(t.sess.seq_ids, dtype=torch.int32, device="cuda")
+    kd.kv_cache_device_steps(h, B, True, stream)
+    ins = [wl.step_inputs(cfg, 0, l, "cuda") for l in range(L)]
+    outs = [torch.empty_like(x[0]) for x in ins]
+
+    def layers():
+        for l in range(L):
+            kd.decode_attention_append(h, l, B, ins[l][0], ins[l][1], ins[l][2], outs[l], 0.0, stream)
+
+    with torch.cuda.stream(stream):
+        kd.kv_begin_step_device(h, B, ids, stream)
+        layers()
+    stream.synchronize()
+    g_step, g_a, g_b = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_step, stream=stream):
+        kd.kv_begin_step_device(h, B, ids, stream)
+    with torch.cuda.graph(g_a, stream=stream):
+        layers()
+    with torch.cuda.graph(g_b, stream=stream):
+        layers()
+
+    def timed(g):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g_step.replay()
+                g.replay()
+            ev[0].record(stream)
+            for _ in range(10):
+                g_step.replay()
+                g.replay()
+            ev[1].record(stream)
+        stream.synchronize()
+        return ev[0].elapsed_time(ev[1]) / 10
+
+    ta, tb = timed(g_a), timed(g_b)
+    assert tb < 2 * ta + 0.05, (ta, tb)
+    st = kd.kv_cache_query(h)
+    assert st.device_error == 0
+    t.close()
