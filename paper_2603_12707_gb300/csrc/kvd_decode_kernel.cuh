@@ -392,20 +392,36 @@ struct GqaCompute {
     }
 };
 
-// The new token of row (en.b, g) into row r of the staged K and V tiles and,
-// unless its page id is out of range (already recorded), into the pool
-// (fused append): lanes 0..CH-1 move K, CH..2CH-1 move V.
+// The new token of row (en.b, g), 16 bytes per lane: lanes 0..CH-1 hold K,
+// CH..2CH-1 hold V.  Loaded when the row's last item starts, so the load is
+// back long before its last page (where waiting for it cost ~2 us under a
+// saturated HBM).
+template <int D>
+__device__ __forceinline__ uint4 load_new_token(const DecodeParams& p, const PlanEntry& en, int g, int lane)
+{
+    constexpr int CH = D / 8;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (lane < 2 * CH) {
+        const bool is_k = lane < CH;
+        const int c = is_k ? lane : lane - CH;
+        const int64_t src = ((int64_t)en.b * p.H_kv + g) * D + c * 8;
+        v = *reinterpret_cast<const uint4*>((is_k ? p.k_new : p.v_new) + src);
+    }
+    return v;
+}
+
+// The new token (load_new_token's v) into row r of the staged K and V tiles
+// and, unless its page id is out of range (already recorded), into the pool
+// (fused append).
 template <int D>
 __device__ __forceinline__ void put_new_token(const DecodeParams& p, const PlanEntry& en, int g, int32_t pid,
-                                              uint8_t* sK, uint8_t* sV, int lane)
+                                              const uint4& v, uint8_t* sK, uint8_t* sV, int lane)
 {
     constexpr int CH = D / 8;
     const int r = (en.len - 1) % kPageSize;
     if (lane < 2 * CH) {
         const bool is_k = lane < CH;
         const int c = is_k ? lane : lane - CH;
-        const int64_t src = ((int64_t)en.b * p.H_kv + g) * D + c * 8;
-        const uint4 v = *reinterpret_cast<const uint4*>((is_k ? p.k_new : p.v_new) + src);
         *reinterpret_cast<uint4*>((is_k ? sK : sV) + swz(r, c)) = v;
         if (pid >= 0 && pid < p.num_pages) {
             const int64_t dst = (((int64_t)pid * p.H_kv + g) * kPageSize + r) * D + c * 8;
@@ -540,6 +556,10 @@ __global__ void __launch_bounds__(kWarps * 32)
         }
         first_item = false;
         comp.start(p, en, g, lane);
+        const bool last_chunk = en.chunk == en.n_chunks - 1;
+        uint4 new_kv = make_uint4(0u, 0u, 0u, 0u);
+        if constexpr (FUSED)
+            if (last_chunk) new_kv = load_new_token<D>(p, en, g, lane);
 
         for (int j = 0; j < np; ++j) {
             const int s = j % R;
@@ -558,9 +578,9 @@ __global__ void __launch_bounds__(kWarps * 32)
             bool wrote = GQA && valid < kPageSize;
             if constexpr (FUSED) {
                 // the issue side has not moved past this page's id window
-                if (en.chunk == en.n_chunks - 1 && j == np - 1) {
+                if (last_chunk && j == np - 1) {
                     int32_t pid = __shfl_sync(0xffffffffu, pid_cur, j & 31);
-                    put_new_token<D>(p, en, g, pid, sK, sK + TILE, lane);
+                    put_new_token<D>(p, en, g, pid, new_kv, sK, sK + TILE, lane);
                     wrote = true;
                 }
             }
