@@ -251,7 +251,7 @@ struct GqaCompute {
             for (int k = 0; k < 4; ++k) oacc[mt][k] = 0.f;
     }
 
-    __device__ __forceinline__ void page(uint8_t*, uint8_t* sVp, uint32_t sK, uint32_t sV, int valid,
+    __device__ __forceinline__ void page(uint8_t*, uint8_t*, uint32_t sK, uint32_t sV, int valid,
                                          float scale_log2, int lane)
     {
         // S^T over the D/16 k-steps in four independent accumulator chains
@@ -275,6 +275,30 @@ struct GqaCompute {
             for (int a = 0; a < NA; ++a)
 #pragma unroll
                 for (int k = 0; k < 4; ++k) sc[k] += acc[a][k];
+        }
+        // V^T's fragments now, so their shared-memory latency overlaps the
+        // softmax.  Rows past the end may hold anything (a NaN pattern would
+        // survive a zero weight), so a partial page zeroes their bf16 halves
+        // in registers: lane t holds tokens 2(t%4), 2(t%4)+1 in a0/a1 and
+        // those + 8 in a2/a3.
+        uint32_t vf[KS][4];
+        {
+            const int r = (lane & 7) + (lane >> 4) * 8;
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt)
+                ldsm_x4_trans(sV + swz(r, mt * 2 + ((lane >> 3) & 1)), vf[mt][0], vf[mt][1], vf[mt][2], vf[mt][3]);
+            if (valid < kPageSize) {
+                const int tk = 2 * (lane & 3);
+                const uint32_t ma = (tk < valid ? 0x0000ffffu : 0u) | (tk + 1 < valid ? 0xffff0000u : 0u);
+                const uint32_t mb = (tk + 8 < valid ? 0x0000ffffu : 0u) | (tk + 9 < valid ? 0xffff0000u : 0u);
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                    vf[mt][0] &= ma;
+                    vf[mt][1] &= ma;
+                    vf[mt][2] &= mb;
+                    vf[mt][3] &= mb;
+                }
+            }
         }
         const int t0 = lane >> 2, t1 = t0 + 8;
         const bool v0 = t0 < valid, v1 = t1 < valid;
@@ -314,35 +338,14 @@ struct GqaCompute {
         l0 += p0 + p2;
         l1 += p1 + p3;
         // P^T as the B operand: lane needs P[t=2(lane&3)+{0,1}][h=lane>>2] and
-        // the same for t+8.  P[t][h] for t < 8 sits in lane 4t + h/2.
-        const int srcA = 8 * (lane & 3) + (lane >> 3);
-        const int srcB = srcA + 4;
-        const uint32_t u01 = pack_bf16(p0, p1), u23 = pack_bf16(p2, p3);
-        const uint32_t xa = __shfl_sync(0xffffffffu, u01, srcA);
-        const uint32_t xb = __shfl_sync(0xffffffffu, u01, srcB);
-        const uint32_t za = __shfl_sync(0xffffffffu, u23, srcA);
-        const uint32_t zb = __shfl_sync(0xffffffffu, u23, srcB);
-        const uint32_t sel = ((lane >> 2) & 1) ? 0x7632u : 0x5410u;
-        const uint32_t pb0 = __byte_perm(xa, xb, sel);
-        const uint32_t pb1 = __byte_perm(za, zb, sel);
-
-        if (valid < kPageSize) {   // rows past the end may hold anything
-            constexpr int CH = D / 8;
-            for (int i = lane; i < (kPageSize - valid) * CH; i += 32) {
-                const int r = valid + i / CH;
-                *reinterpret_cast<uint4*>(sVp + swz(r, i % CH)) = make_uint4(0, 0, 0, 0);
-            }
-            __syncwarp();
-        }
-        {
-            const int r = (lane & 7) + (lane >> 4) * 8;
+        // the same for t+8.  The packed accumulator pairs (tokens 0-7, then
+        // 8-15) are 8x8 bf16 tiles [token][head] in the m8n8 fragment layout;
+        // their transposes are the B fragments.
+        const uint32_t pb0 = movmatrix_trans(pack_bf16(p0, p1));
+        const uint32_t pb1 = movmatrix_trans(pack_bf16(p2, p3));
 #pragma unroll
-            for (int mt = 0; mt < KS; ++mt) {
-                uint32_t a0, a1, a2, a3;
-                ldsm_x4_trans(sV + swz(r, mt * 2 + ((lane >> 3) & 1)), a0, a1, a2, a3);
-                mma_bf16_16816(oacc[mt], a0, a1, a2, a3, pb0, pb1);
-            }
-        }
+        for (int mt = 0; mt < KS; ++mt)
+            mma_bf16_16816(oacc[mt], vf[mt][0], vf[mt][1], vf[mt][2], vf[mt][3], pb0, pb1);
     }
 
     __device__ __forceinline__ void finish(const DecodeParams& p, const PlanEntry& en, int g, int lane)
@@ -572,10 +575,10 @@ __global__ void __launch_bounds__(kWarps * 32)
             pending &= ~(1u << s);
             const int valid = min(kPageSize, en.len - (en.first_page + j) * kPageSize);
             uint8_t* sK = ring + s * STAGE;
-            // Generic-proxy writes into the stage (the new token's row, zeroed
-            // rows past the end) must be ordered before the next TMA write to
-            // it; plain reads need no fence (their values are consumed first).
-            bool wrote = GQA && valid < kPageSize;
+            // Generic-proxy writes into the stage (the new token's row) must be
+            // ordered before the next TMA write to it; plain reads need no
+            // fence (their values are consumed first).
+            bool wrote = false;
             if constexpr (FUSED) {
                 // the issue side has not moved past this page's id window
                 if (last_chunk && j == np - 1) {

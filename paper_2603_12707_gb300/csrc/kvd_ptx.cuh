@@ -1,5 +1,5 @@
 // Inline-PTX helpers for sm_103a: mbarrier, 3-D / 4-D TMA tile loads, ldmatrix,
-// warp-level bf16 MMA, ex2, bf16 packing.
+// movmatrix, warp-level bf16 MMA, ex2, bf16 packing.
 #pragma once
 
 #include <cuda.h>
@@ -155,6 +155,15 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint3
         "{%8,%9}, {%0,%1,%2,%3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Transpose of an 8x8 b16 tile held in the m8n8 fragment layout (lane t
+// holds row t/4, columns 2(t%4) and 2(t%4)+1).
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a)
+{
+    uint32_t d;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+    return d;
 }
 
 // ---- scalar helpers ---------------------------------------------------------------
