@@ -119,3 +119,34 @@ def assert_close(got, ref, vmax, gqa: bool, what=""):
     bound = 2.0 ** -8 * np.abs(ref) + w * vmax[:, None, None]
     bad = err > bound
     assert not bad.any(), (what, int(bad.sum()), float((err - bound).max()), np.argwhere(bad)[:5].tolist())
+
+
+# NaN, -NaN, +Inf and -Inf as bf16 bit patterns (int16 view)
+POISON = (0x7FC0, 0xFFC0 - 0x10000, 0x7F80, 0xFF80 - 0x10000)
+
+
+def poison_unused_slots(sess: DecodeSession):
+    """Fill every pool slot that no sequence holds (the free pages, and the
+    slots past each sequence's length on its last page) with NaN / Inf bit
+    patterns in every layer's K and V pools, so a result that let one of them
+    in shows it.  Returns the number of slots poisoned per pool."""
+    c = sess.cfg
+    P = c.page_size
+    used = np.zeros((sess.num_pages, P), bool)
+    for seq in sess.seq_ids:
+        n, pages = kd.kv_seq_info(sess.h, seq)
+        for i, pg in enumerate(pages):
+            k = min(P, n - i * P)
+            if k > 0:
+                used[pg, :k] = True
+    idx = np.arange(sess.num_pages)[:, None] + np.arange(P)[None, :]
+    patt = np.array(POISON, np.int16)[idx % len(POISON)]
+    mask = torch.from_numpy(~used).cuda()[:, None, :, None]
+    fill = torch.from_numpy(patt).cuda()[:, None, :, None]
+    shape = (sess.num_pages, c.num_kv_heads, P, c.head_dim)
+    for layer in range(c.phys_layers):
+        for ptr in kd.kv_cache_pool(sess.h, layer):
+            pool = torch.as_tensor(_CAI(ptr, shape), device="cuda")
+            pool.copy_(torch.where(mask, fill, pool))
+    torch.cuda.synchronize()
+    return int((~used).sum())

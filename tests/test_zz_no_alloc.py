@@ -4,8 +4,8 @@ at build time, a runtime whose device memory belongs to another framework's
 allocator).  It runs on a 16 MiB static scratch array instead of cache-owned
 buffers.  Checked here: its output against decode_attention's on the same
 cache contents and against the float64 oracle reading the same pools through
-the same page table, on two calls in a row (the second reuses the scratch the
-first left behind); a batch whose plan only fits the scratch after the item
+the same page table, with NaN / Inf patterns in every pool slot no row holds,
+on two calls in a row (the second reuses the scratch the first left behind); a batch whose plan only fits the scratch after the item
 size has doubled; a batch that never fits (KVC_ERR_UNSUPPORTED); argument
 checks.  This file is collected last on purpose."""
 import numpy as np
@@ -16,7 +16,7 @@ import oracle
 from paper_2603_12707_gb300 import kvdecode as kd
 from paper_2603_12707_gb300 import workloads as wl
 
-from _gpu_common import Tracked, assert_close, bf16_to_f64, device_pool, u16
+from _gpu_common import Tracked, assert_close, bf16_to_f64, device_pool, poison_unused_slots, u16
 
 pytestmark = pytest.mark.gpu
 
@@ -49,6 +49,7 @@ def test_noalloc_matches_decode_attention_and_oracle_on_two_calls(kvlib, Hq, Hkv
     cfg = wl.custom("noalloc", 2, Hq, Hkv, d, len(lens), lens=lens, seed=17 + Hq, page_order="shuffled")
     t = Tracked(cfg, keep_host=False)
     sess = t.sess
+    poison_unused_slots(sess)      # NaN / Inf in every slot no row holds
     t.begin_step()
     out_ref, q, _, _ = t.run_layer(1)
     pt = _page_table(sess)
