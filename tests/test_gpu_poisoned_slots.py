@@ -4,8 +4,9 @@ left there.  Every such slot, in every layer's K and V pools, is filled here
 with NaN and Inf bit patterns before the steps run; the partial last page of
 a row (and the page an append opens) then carries them in its rows past the
 row's length.  The outputs must stay finite and match the float64 oracle,
-which sees only the tokens each row holds, for MHA and GQA, head dims 64 and
-128, fused and unfused launches, and item sizes from one page up."""
+which sees only the tokens each row holds, for MHA and every GQA group size
+(2 to 8), head dims 64 and 128, fused and unfused launches, and item sizes
+from one page up."""
 import numpy as np
 import pytest
 import torch
@@ -30,6 +31,11 @@ def _lib(kvlib):
     ("gqa3_128", 12, 4, 128, [2, 32, 47]),
     ("mha64", 8, 8, 64, [5, 16, 129]),
     ("gqa8_64", 16, 2, 64, [1, 15, 48, 99]),
+    ("gqa2_64", 8, 4, 64, [3, 31, 64]),
+    ("gqa4_128", 16, 4, 128, [9, 16, 70]),
+    ("gqa5_128", 20, 4, 128, [1, 18, 45]),
+    ("gqa6_64", 24, 4, 64, [7, 32, 81]),
+    ("gqa8_128", 32, 4, 128, [2, 17, 150]),
 ])
 def test_nan_and_inf_in_unheld_slots_never_reach_the_output(name, Hq, Hkv, d, lens, split):
     cfg = wl.custom(name, 2, Hq, Hkv, d, len(lens), lens=lens, seed=71 + Hq + d, page_order="shuffled")
