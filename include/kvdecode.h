@@ -114,9 +114,9 @@ KVC_API int kv_cache_destroy(kv_cache *cache);
  * 0 .. num_pages-1, and no page may be in use. */
 KVC_API int kv_cache_set_page_order(kv_cache *cache, const int32_t *order, int64_t n);
 
-/* Wait for the cache's stream (the stream of its latest call; the whole
- * device if that stream has been destroyed since) and report usage and
- * device error bits, read back on a stream the cache owns.  Returns
+/* Wait for the cache's stream (the stream of its latest call, which must
+ * still exist; should waiting on it fail, the whole device) and report usage
+ * and device error bits, read back on a stream the cache owns.  Returns
  * KVC_ERR_PAGE_TABLE (page or length range), KVC_ERR_OOM (a device-side step
  * ran out of pages) or KVC_ERR_DEVICE (a pipeline wait gave up) if
  * device_error is non-zero; the stats are filled in either way. */
@@ -277,9 +277,9 @@ KVC_API int decode_attention_append(kv_cache *cache, int32_t layer, int32_t batc
  * by the next call that reads it (kv_seq_info, kv_begin_step,
  * kv_cache_query, kv_cache_set_page_order, kv_cache_device_steps or
  * kv_cache_sync), which waits for the cache's stream (the stream of the
- * cache's latest call, so replay the graphs on that stream; the whole device
- * if it has been destroyed since) and reads the state back on a stream the
- * cache owns.  Graphs captured while device
+ * cache's latest call, so replay the graphs on that stream; it must still
+ * exist, and should waiting on it fail, the whole device) and reads the
+ * state back on a stream the cache owns.  Graphs captured while device
  * steps are enabled stay valid until they are disabled, enabled again (which
  * may resize the buffers) or the cache is destroyed: meanwhile a host-planned
  * step that would need larger buffers fails with KVC_ERR_INVALID instead of
@@ -297,8 +297,9 @@ KVC_API int kv_cache_device_steps(kv_cache *cache, int32_t max_batch, int32_t en
  * host synchronisation; graph-capturable. */
 KVC_API int kv_begin_step_device(kv_cache *cache, int32_t batch, const int32_t *seq_ids, void *stream);
 
-/* Wait for the cache's stream (the stream of its latest call) and refresh the
- * host allocator's view after device-side steps and allocator calls. */
+/* Wait for the cache's stream (the stream of its latest call, which must
+ * still exist) and refresh the host allocator's view after device-side steps
+ * and allocator calls. */
 KVC_API int kv_cache_sync(kv_cache *cache);
 
 /* ------------------------------------------------ allocation-free decode -- */

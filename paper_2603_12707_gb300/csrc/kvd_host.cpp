@@ -273,8 +273,8 @@ void release_device(kv_cache* c)
     cudaFree(c->part_ml);
 }
 
-// Wait for the cache's stream (the stream of its latest call).  Should that
-// handle no longer be a stream (the caller destroyed it), wait for the device.
+// Wait for the cache's stream (the stream of its latest call; the caller
+// keeps it alive).  Should the wait fail, wait for the device instead.
 int wait_cache_stream(kv_cache* c)
 {
     if (cudaStreamSynchronize(c->last_stream) != cudaSuccess) {
