@@ -97,6 +97,10 @@ SMALL = [
     ("gqa5_128", 10, 2, 128, [1, 48, 511]),
     ("gqa6_64", 12, 2, 64, [9, 80, 257]),
     ("gqa8_128", 8, 1, 128, [31, 250, 1100]),
+    # the head shapes of the larger backends in the paper's footprint table (Table 3):
+    # LLaVA-13B (MHA 40/40) and LLaVA-34B (GQA 56 query heads over 8 KV heads), d 128
+    ("llava13b", 40, 40, 128, [7, 16, 577, 1200]),
+    ("llava34b", 56, 8, 128, [1, 32, 640, 2000]),
     # rows longer than a 32-page id window, and longer than the item cap at small splits
     ("mha64_long", 8, 8, 64, [3000, 40]),
     ("gqa7_long", 28, 4, 128, [4000, 5]),
