@@ -44,6 +44,7 @@ def _close(got, ref, vmax, gqa):
     (32, 32, 128, [700, 1, 16, 17, 1300, 95]),
     (28, 4, 128, [2048, 300, 33, 5000]),
     (8, 8, 64, [96, 96, 96, 96]),
+    (16, 2, 64, [1, 250, 31, 700, 16]),
 ])
 def test_noalloc_matches_decode_attention_and_oracle_on_two_calls(kvlib, Hq, Hkv, d, lens):
     cfg = wl.custom("noalloc", 2, Hq, Hkv, d, len(lens), lens=lens, seed=17 + Hq, page_order="shuffled")
