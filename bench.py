@@ -73,6 +73,11 @@ def layer_bytes(cfg, attended):
     return attn, app
 
 
+def kv_bytes(cfg, attended):
+    """KV bytes one layer reads for the attended lengths."""
+    return int(sum(attended)) * 2 * cfg.num_kv_heads * cfg.head_dim * 2
+
+
 def describe(cfg):
     return {"workload": cfg.name + ": " + cfg.description, "batch": cfg.batch, "layers": cfg.num_layers,
             "layer_pools": cfg.phys_layers, "q_heads": cfg.num_q_heads, "kv_heads": cfg.num_kv_heads,
@@ -385,7 +390,9 @@ def run_gpu(args, rank, world, cfg):
             step_bytes.append(L * (a + p))
             attn_bytes.append(a if args.unfused else a + p)   # the fused kernel also writes the new K/V
         return {"ms": step_ev[0].elapsed_time(step_ev[-1]), "step_ms": step_ms, "attn_ms": attn_ms,
-                "step_bytes": step_bytes, "attn_bytes": attn_bytes}
+                "step_bytes": step_bytes, "attn_bytes": attn_bytes,
+                "attended": [statistics.mean(att) for att in attended],
+                "kv_bytes": [L * kv_bytes(cfg, att) for att in attended]}
 
     for attempt in range(2):
         if world > 1:
@@ -496,10 +503,12 @@ def run_gpu(args, rank, world, cfg):
         st = sess.query()
         assert st.device_error == 0
 
+    start_attended = statistics.mean(int(n) for n in sess.lens0) + 1   # the first step's contexts
     sess.close()
     del sess
     torch.cuda.synchronize()
-    return {"blocks": blocks, "launches": timed_launches, "clocks": clock_summary, "e2e": e2e, "cfg": cfg, "L": L}
+    return {"blocks": blocks, "launches": timed_launches, "clocks": clock_summary, "e2e": e2e, "cfg": cfg, "L": L,
+            "start_attended": start_attended}
 
 
 def run_varlen_write(args, rank, world):
@@ -745,6 +754,12 @@ def summarize(args, world, r):
                    "parallelism": f"replicas x{world}"},
         "steps_per_s": round(args.steps / (ms / 1e3), 3),
         "timed_blocks": len(blocks),
+        # every step appends a token, so the blocks attend longer contexts as the
+        # run goes on: the median block's workload, for reading the numbers above
+        "median_block_context": {"mean_attended_tokens": round(statistics.mean(mid["attended"]), 1),
+                                 "kv_gb_per_step": round(statistics.mean(mid["kv_bytes"]) / 1e9, 4),
+                                 "tokens_appended_before_it": int(round(statistics.mean(mid["attended"])
+                                                                        - r["start_attended"]))},
         "block_statistic": f"median of {len(blocks)} consecutive timed blocks of {args.steps} steps each "
                            "(contexts grow by one token per step across the blocks)",
         "block_ms": [round(b["ms"], 4) for b in blocks],

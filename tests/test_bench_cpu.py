@@ -6,6 +6,7 @@ import argparse
 import json
 import os
 import shutil
+import statistics
 import sys
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -130,11 +131,15 @@ def _fake_run(cfg, block_ms, steps, L):
             attn_bytes.append(a + p)
             lens = [n + 1 for n in lens]
         blocks.append({"ms": ms, "step_ms": [ms / steps] * steps, "attn_ms": [0.9 * ms / steps / L] * steps,
-                       "step_bytes": step_bytes, "attn_bytes": attn_bytes})
+                       "step_bytes": step_bytes, "attn_bytes": attn_bytes,
+                       "attended": [150.5 + len(blocks) * steps + i for i in range(steps)],
+                       "kv_bytes": [L * bench.kv_bytes(cfg, [101 + len(blocks) * steps + i, 201 + len(blocks) * steps + i])
+                                    for i in range(steps)]})
     clocks = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 12, "retimed": False}
     e2e = {"ms": 1.1 * sum(block_ms) / len(block_ms), "wall_s": 0.1, "bytes": sum(blocks[0]["step_bytes"]),
            "h2d": 1000, "d2h": 500}
-    return {"blocks": blocks, "launches": 3 * steps, "clocks": clocks, "e2e": e2e, "cfg": cfg, "L": L}
+    return {"blocks": blocks, "launches": 3 * steps, "clocks": clocks, "e2e": e2e, "cfg": cfg, "L": L,
+            "start_attended": 151.0}
 
 
 def test_summary_reports_the_median_block_and_every_contract_key():
@@ -159,3 +164,9 @@ def test_summary_reports_the_median_block_and_every_contract_key():
     assert out["e2e"]["unit"] == "GB/s" and out["e2e"]["value"] > 0
     assert out["clocks"]["samples"] == 12 and out["gpu_launches"] == 3 * steps
     assert out["config"]["workload"].startswith("fake") and "l2" in out["config"]
+    # the median block (the third) attends 158.5 .. 161.5 tokens on average over its steps
+    ctx = out["median_block_context"]
+    assert ctx["mean_attended_tokens"] == 160.0
+    assert ctx["tokens_appended_before_it"] == 9
+    kv = statistics.mean(L * bench.kv_bytes(cfg, [109 + i, 209 + i]) for i in range(steps))
+    assert ctx["kv_gb_per_step"] == round(kv / 1e9, 4)
