@@ -104,6 +104,7 @@ SMALL = [
     # rows longer than a 32-page id window, and longer than the item cap at small splits
     ("mha64_long", 8, 8, 64, [3000, 40]),
     ("gqa7_long", 28, 4, 128, [4000, 5]),
+    ("gqa7_64_long", 14, 2, 64, [2600, 33, 700]),   # d 64: a 6-stage ring across id windows
 ]
 
 
