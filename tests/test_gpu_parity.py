@@ -115,8 +115,9 @@ def test_merge_batch_variants(Hq, Hkv, d, max_items):
     launch picks the smallest that covers the step's longest row: one-page
     items and a longest row of max_items pages exercise each variant, with
     shorter rows (one item, several items) beside it.  These batches have
-    few rows, so rows may hold up to 64 items: 48 and 64 exercise the second
-    (m, l) per lane and a second batch of loads."""
+    few rows, so rows may hold up to 64 items: 48 and 64 take the four-warp
+    variant (16 items per warp, combined in shared memory), one with an idle
+    warp."""
     lens = [16 * max_items - 1, 40, 5, 16 * max(1, max_items // 2)]
     cfg = wl.custom(f"merge{max_items}", 1, Hq, Hkv, d, len(lens), lens=lens, seed=400 + max_items,
                     page_order="shuffled")
