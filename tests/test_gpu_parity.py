@@ -108,16 +108,16 @@ SMALL = [
 ]
 
 
-@pytest.mark.parametrize("max_items", [2, 3, 7, 12, 20, 32, 48, 64])
+@pytest.mark.parametrize("max_items", [2, 3, 7, 12, 20, 32, 33, 48, 64])
 @pytest.mark.parametrize("Hq,Hkv,d", [(8, 8, 128), (28, 4, 128), (14, 2, 64)])
 def test_merge_batch_variants(Hq, Hkv, d, max_items):
     """The merge pass is compiled for 4, 8, 16 or 32 items in flight and the
     launch picks the smallest that covers the step's longest row: one-page
     items and a longest row of max_items pages exercise each variant, with
     shorter rows (one item, several items) beside it.  These batches have
-    few rows, so rows may hold up to 64 items: 48 and 64 take the four-warp
-    variant (16 items per warp, combined in shared memory), one with an idle
-    warp."""
+    few rows, so rows may hold up to 64 items: 33, 48 and 64 take the
+    four-warp variant (16 items per warp, combined in shared memory; at 33 a
+    warp with one item and an idle warp)."""
     lens = [16 * max_items - 1, 40, 5, 16 * max(1, max_items // 2)]
     cfg = wl.custom(f"merge{max_items}", 1, Hq, Hkv, d, len(lens), lens=lens, seed=400 + max_items,
                     page_order="shuffled")
