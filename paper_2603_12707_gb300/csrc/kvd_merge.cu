@@ -144,6 +144,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) merge_kernel(const DecodePar
 // and weighs 0), in one round trip where a single warp would need two.
 constexpr int kWideWarps = 4;
 constexpr int kWideItems = 16;   // items per warp
+static_assert(kWideWarps * kWideItems >= kMaxChunks, "a row's items (at most kMaxChunks) fit one CTA");
 
 template <int D>
 __global__ void __launch_bounds__(kWideWarps * 32) merge_wide_kernel(const DecodeParams p, int pdl)
